@@ -1,0 +1,233 @@
+/*
+ * kvtier.h - C ABI of the hot/cold KV tiering hot path for one GB300 GPU.
+ *
+ * The library implements the data paths of the hot-cold KV hierarchy of
+ * Baek et al., "Hot-Cold Tiering of HBM and High Bandwidth Flash for Agentic
+ * LLM Serving" (Section 3, "Architecture and data paths"):
+ *   path 1  decode attention over the HBM-resident hot set ... decode_attention
+ *   path 2  resume: cold image -> hot blocks ................ session_resume
+ *   path 3  fresh KV written into hot blocks ................ session_append
+ *   path 4  eviction: hot blocks -> cold image .............. session_pause
+ * The cold tier (high bandwidth flash in the paper) is a second device
+ * allocation; its bandwidth, energy and endurance are not modelled.
+ *
+ * Data layout (all bf16, D = head_dim = 128, bt = block_tokens):
+ *   hot pool   hot[num_hot_blocks][L][2][Hkv][bt][D]   (2 = K, V)
+ *              One block holds bt tokens of every layer: 16 tokens x 96 KiB
+ *              = 1.5 MiB for L=48, Hkv=4 (the paper's block unit, Section 4).
+ *              Each (block, layer, K|V, kv-head) run is bt*D*2 = 4 KiB.
+ *   cold image img[L][2][Hkv][T_cap][D] per session, contiguous and
+ *              layer-major, placed in the cold arena by the pool.
+ *   block table: row of int32 physical block ids; logical block j of a
+ *              session holds its tokens j*bt .. j*bt+bt-1.
+ *
+ * Conventions for every call:
+ *  - Return value 0 (KV_OK) or a negative KV_ERR_* code. On error nothing
+ *    changes: no host state, no block ownership, no device work enqueued
+ *    that would alter data. kv_last_error() describes the last failure of
+ *    the calling thread.
+ *  - Pointers documented as "device" are CUDA device addresses on the pool's
+ *    device; "host" pointers are ordinary CPU memory read or written before
+ *    the call returns.
+ *  - Device work is enqueued on the given stream and is asynchronous; host
+ *    metadata (states, lengths, tables, the free list) changes when the call
+ *    returns. Streams are cudaStream_t values (kv_stream_t is the same type);
+ *    0 is the legacy default stream.
+ *  - The caller owns the hot and cold arenas, Q, outputs, batch tables and
+ *    streams. The pool owns its metadata, a device block-table arena, the
+ *    decode workspace and its CUDA events.
+ *  - A pool is not thread-safe: one host thread at a time.
+ */
+#ifndef KVTIER_H
+#define KVTIER_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *kv_stream_t; /* == cudaStream_t */
+typedef struct CUevent_st *kv_event_t;   /* == cudaEvent_t  */
+typedef struct kv_pool kv_pool;          /* opaque */
+
+enum {
+    KV_OK = 0,
+    KV_ERR_INVALID_ARG = -1,   /* bad size, pointer, id or shape */
+    KV_ERR_BAD_STATE = -2,     /* e.g. resume of an active session */
+    KV_ERR_NO_HOT_BLOCKS = -3, /* free list cannot cover the request */
+    KV_ERR_NO_COLD_SPACE = -4, /* cold arena cannot hold the image */
+    KV_ERR_CUDA = -5,          /* a CUDA runtime call failed */
+    KV_ERR_DEVICE_CHECK = -6   /* a kernel's own bounds check fired */
+};
+
+enum { KV_SESSION_FREE = 0, KV_SESSION_ACTIVE = 1, KV_SESSION_PAUSED = 2 };
+
+/* Pool flag: bookkeeping only. No CUDA call is made, no kernel runs and no
+ * data moves; calls that would compute return KV_ERR_BAD_STATE. Used to test
+ * the host logic (placement, states, errors) on machines without a GPU. */
+#define KV_POOL_HOST_LOGIC_ONLY 1u
+
+typedef struct kv_pool_config {
+    int32_t num_layers;     /* L  (48 for Qwen3-Coder-30B-A3B)             */
+    int32_t num_q_heads;    /* Hq (32); Hq / Hkv must be 1, 2, 4 or 8      */
+    int32_t num_kv_heads;   /* Hkv (4), at most 8                          */
+    int32_t head_dim;       /* D; must be 128                              */
+    int32_t block_tokens;   /* bt; 16 or 64                                */
+    int32_t max_sessions;   /* session ids are 0 .. max_sessions-1          */
+    int32_t max_batch;      /* largest B passed to decode_attention         */
+    int32_t device;         /* CUDA ordinal holding both arenas             */
+    int64_t max_context;    /* longest session in tokens (table width)      */
+    int64_t num_hot_blocks; /* blocks in the hot arena                      */
+    void *hot_base;         /* device, >= num_hot_blocks * block bytes, 256-B aligned */
+    int64_t cold_bytes;     /* bytes in the cold arena                      */
+    void *cold_base;        /* device, 256-B aligned                        */
+    uint64_t alloc_seed;    /* seeds the shuffle of the initial free list   */
+    uint32_t flags;         /* 0 or KV_POOL_HOST_LOGIC_ONLY                 */
+    uint32_t reserved;
+} kv_pool_config;
+
+typedef struct kv_session_info {
+    int32_t state;       /* KV_SESSION_*                                   */
+    int32_t num_blocks;  /* hot blocks held (0 when paused)                */
+    int64_t tokens;      /* T: tokens in the session's KV                  */
+    int64_t capacity;    /* T_cap of its cold image                        */
+    int64_t cold_valid;  /* tokens already valid in the cold image         */
+    void *image;         /* device address of img[L][2][Hkv][T_cap][D]     */
+} kv_session_info;
+
+typedef struct kv_pool_stats {
+    int64_t free_blocks;
+    int64_t used_blocks;
+    int64_t cold_bytes_used;
+    int64_t bytes_unpacked;   /* image bytes copied cold -> hot (path 2)   */
+    int64_t bytes_packed;     /* image bytes copied hot -> cold (path 4)   */
+    int64_t bytes_appended;   /* KV bytes written by session_append        */
+    int64_t resumes, pauses, appends, decodes;
+} kv_pool_stats;
+
+/* Create a pool over caller-owned arenas. The hot free list starts as
+ * 0..num_hot_blocks-1 shuffled by Fisher-Yates driven by splitmix64 seeded
+ * with alloc_seed (draw j = floor(r * (i+1) / 2^64) for i = n-1 .. 1);
+ * allocations pop from its end. *out receives the pool. */
+int kv_pool_create(const kv_pool_config *cfg, kv_pool **out);
+
+/* Destroy a pool after synchronising its device. Arenas are not freed. */
+int kv_pool_destroy(kv_pool *pool);
+
+/* Bytes of one hot block: L * 2 * Hkv * bt * D * 2. */
+int64_t kv_block_bytes(const kv_pool_config *cfg);
+
+/* Bytes of K plus V per token: L * 2 * Hkv * D * 2 (96 KiB for the paper's
+ * model, Section 4). */
+int64_t kv_token_bytes(const kv_pool_config *cfg);
+
+/* Create an ACTIVE, empty session able to hold max_tokens (1 ..
+ * max_context) tokens; reserves its cold image (max_tokens * token bytes)
+ * in the cold arena (first fit). Errors: KV_ERR_NO_COLD_SPACE, too many
+ * sessions -> KV_ERR_INVALID_ARG. */
+int session_create(kv_pool *pool, int64_t max_tokens, int32_t *sid_out);
+
+/* Create a PAUSED session whose image the caller fills with `tokens` valid
+ * tokens (session_info gives its device address); cold_valid = tokens. */
+int session_create_paused(kv_pool *pool, int64_t max_tokens, int64_t tokens,
+                          int32_t *sid_out);
+
+/* Release a session's hot blocks and cold image (any state). The caller
+ * must have finished all work that reads them. */
+int session_destroy(kv_pool *pool, int32_t sid);
+
+/* Data path 3 (Section 3): write n >= 1 new tokens of an ACTIVE session.
+ * k, v: device, bf16 [L][n][Hkv][D] contiguous. Blocks are popped from the
+ * free list when the tail block fills; tokens go to positions T .. T+n-1,
+ * then T += n. The stream first waits for the session's last resume.
+ * Errors: KV_ERR_BAD_STATE (paused), KV_ERR_NO_HOT_BLOCKS, capacity
+ * exceeded -> KV_ERR_INVALID_ARG. */
+int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int32_t n,
+                   kv_stream_t stream);
+
+/* Data path 1 (Section 3; Section 2: decoding attends to the cached KV):
+ * one decode step of grouped-query attention for B sessions.
+ *   layer        0 .. L-1, or -1 for all layers in one launch (q and out
+ *                then carry a leading [L] dimension)
+ *   q            device bf16 [B][Hq][D]   (or [L][B][Hq][D])
+ *   block_tables device int32 [B][max_blocks]; row b lists session b's
+ *                blocks in logical order
+ *   seq_lens     device int32 [B]; 1 <= seq_lens[b] <= max_blocks * bt
+ *   scale        multiplies q.k before the softmax (1/sqrt(D) usually)
+ *   out          device fp32 [B][Hq][D]   (or [L][B][Hq][D])
+ * out[b][h] = sum_i softmax_i(scale * q[b][h] . K[g][i]) V[g][i] over the
+ * session's tokens i < seq_lens[b], g = h / (Hq/Hkv). Tokens past seq_len
+ * in the last block are never read into the result (they may hold NaN).
+ * The result depends only on the values and seq_lens: not on physical
+ * placement, batch composition or timing (bit-identical across a
+ * pause/resume round trip). B must not exceed max_batch and max_blocks*bt
+ * must not exceed max_context rounded up to a block. */
+int decode_attention(kv_pool *pool, int32_t layer, const void *q,
+                     const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
+                     int32_t max_blocks, float scale, float *out, kv_stream_t stream);
+
+/* Data path 4 with write-on-evict (Section 3, "Memory hierarchy and write
+ * policy"): copy tokens [cold_valid, T) of an ACTIVE session into its
+ * image, set cold_valid = T, return its hot blocks to the end of the free
+ * list in logical order, state -> PAUSED. Tokens already in the image are
+ * not rewritten. The stream first waits for the session's last append; the
+ * caller orders it after any decode that still reads the session. Blocks
+ * are reused only by work ordered after this pack (the pool makes later
+ * allocations wait on its completion event). */
+int session_pause(kv_pool *pool, int32_t sid, kv_stream_t stream);
+
+/* Data path 2 (Section 3, "Eviction, resume and decode"): pop
+ * ceil(T / bt) blocks, write the session's block-table row, copy tokens
+ * [0, T) of its image into them, state -> ACTIVE, and record the session's
+ * ready event on the stream. Errors: KV_ERR_BAD_STATE (not paused),
+ * KV_ERR_NO_HOT_BLOCKS (nothing changes). */
+int session_resume(kv_pool *pool, int32_t sid, kv_stream_t stream);
+
+/* Event recorded after the session's last resume (NULL if none): a decode
+ * stream waits on it before reading the session's blocks. */
+int session_ready_event(kv_pool *pool, int32_t sid, kv_event_t *ev);
+
+/* State, length, capacity, cold_valid and image address of a session. */
+int session_info(kv_pool *pool, int32_t sid, kv_session_info *out);
+
+/* Host copy of a session's block-table row: up to cap entries into
+ * host_row; *nblocks receives the row length. */
+int session_block_table(kv_pool *pool, int32_t sid, int32_t *host_row, int32_t cap,
+                        int32_t *nblocks);
+
+/* Build the decode inputs of a batch of ACTIVE sessions: block_tables
+ * (device int32 [B][max_blocks], entries past a row's length set to -1) and
+ * seq_lens (device int32 [B]) from the pool's tables. sids is a host array
+ * of B ids. */
+int kv_pool_batch_tables(kv_pool *pool, const int32_t *sids, int32_t B, int32_t *block_tables,
+                         int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream);
+
+/* Re-run the Fisher-Yates shuffle over the current free list with a new
+ * seed (scrambles where the next allocations land). */
+int kv_pool_shuffle_free(kv_pool *pool, uint64_t seed);
+
+/* Host copy of the free list (bottom to top): up to cap ids, *n = length. */
+int kv_pool_free_list(kv_pool *pool, int32_t *host_out, int64_t cap, int64_t *n);
+
+int kv_pool_get_stats(kv_pool *pool, kv_pool_stats *out);
+
+/* Synchronise the device and read the flags that kernels set when their own
+ * bounds checks fire (a block id outside the pool, a length past a table
+ * row, a wait that timed out); clears them. *flags = 0 means clean; a
+ * non-zero value makes the call return KV_ERR_DEVICE_CHECK. */
+int kv_pool_check_device(kv_pool *pool, int32_t *flags);
+
+/* Test hook: make the n-th following CUDA call of this pool fail (as a
+ * CUDA error) so tests can check that failing calls change nothing;
+ * n <= 0 disarms. */
+int kv_pool_inject_cuda_failure(kv_pool *pool, int32_t n);
+
+/* Message of the last error on the calling thread ("" if none). */
+const char *kv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVTIER_H */

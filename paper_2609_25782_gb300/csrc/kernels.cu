@@ -1,0 +1,616 @@
+// CUDA kernels of the hot/cold KV tiering hot path, written for sm_103a.
+//
+//   decode_split_kernel    data path 1 (Section 3): split-KV paged GQA decode
+//                          attention with an fp32 online softmax; KV tiles are
+//                          staged by TMA (cp.async.bulk.tensor, 128-byte
+//                          swizzle) into a per-warp mbarrier ring, and the
+//                          group-by-tile products run on mma.sync bf16.
+//   decode_combine_kernel  log-sum-exp merge of the splits, fixed order.
+//   migrate_kernel<false>  data path 2: resume-unpack, cold image -> blocks.
+//   migrate_kernel<true>   data path 4: pause-pack, blocks -> cold image,
+//                          tokens [t0, T) only (write-on-evict, Section 3).
+//   append_kernel          data path 3: fresh tokens into the tail blocks.
+//   table_write_kernel / gather_tables_kernel: block-table bookkeeping.
+//
+// Hot pool: hot[NB][L][2][Hkv][bt][128] bf16. A (block, layer, K|V, head)
+// run is bt rows of 256 B. The decode kernel views the pool as a 2-D tensor
+// of 128-element rows (row = ((blk*L + l)*2 + kv)*Hkv + g)*bt + slot) and
+// loads 16-row x 64-column boxes.
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include "kvt_internal.h"
+
+namespace kvt {
+namespace {
+
+constexpr int kDecodeWarps = 4;
+constexpr int kStages = 3;                 // tiles in flight per warp
+constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
+constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
+constexpr int kDecodeSmem = kDecodeWarps * kStages * kTileBytes + 1024 + 256;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for a phase with a wall-clock limit; false means the limit expired.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                        uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1,
+                                          uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+// D = A(16x16 bf16, row) * B(16x8 bf16, col) + D, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi, float &rlo, float &rhi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    rlo = __low2float(v);
+    rhi = __high2float(v);
+    return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Byte offset, inside a 16-row x 128-byte box written with the 128-byte
+// swizzle, of 16-byte unit `c` (0..7) of row `r`.
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+    return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// ---------------------------------------------------------------------------
+// K1: one CTA = (split s, kv-head g, layer-batch row lb = li*B + b).
+// Warp w consumes the split's tiles w, w+4, ... through its own ring of
+// kStages 8 KiB slots. Per tile (16 tokens):
+//   S^T[16 tok x 8 heads] = K[16 x 128] . Q^T       8 x mma m16n8k16
+//   online softmax over tokens (columns = heads)
+//   O^T[128 x 8] += V^T[128 x 16] . P^T[16 x 8]     8 x mma, P^T via movmatrix
+// The four warps' states merge in shared memory in warp order; a one-split
+// session writes its normalised output, others write (m, l, acc) partials.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kDecodeWarps * 32, 2)
+    decode_split_kernel(const __grid_constant__ CUtensorMap map, const DecodeArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kDecodeWarps * kStages * kTileBytes);
+
+    const int split = blockIdx.x;
+    const int g = blockIdx.y;
+    const int lb = blockIdx.z;
+    const int b = lb % a.B;
+    const int li = lb / a.B;
+    const int l = a.layer0 + li;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const Shape sh = a.s;
+    const int G = sh.Hq / sh.Hkv;
+
+    const int T = a.seq_lens[b];
+    if (T < 1 || T > a.max_blocks * sh.bt) {
+        if (split == 0 && g == 0 && threadIdx.x == 0) atomicOr(a.err, kErrBadLength);
+        return;
+    }
+    const int nsplit = num_splits(T);
+    if (split >= nsplit) return;
+    const int st = split_tiles(T);
+    const int tile0 = split * st;
+    const int tile1 = min(tiles_of(T), tile0 + st);
+    const int my_tiles = (tile1 - tile0 - warp + kDecodeWarps - 1) / kDecodeWarps;  // may be <= 0
+
+    uint8_t *ring = smem + warp * kStages * kTileBytes;
+    const uint32_t ring_s = smem_u32(ring);
+    const uint32_t bar0 = smem_u32(bars + warp * kStages);
+    const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
+    const int chunk_rows = sh.Hkv * sh.bt;   // rows between K and V runs
+
+    if (lane == 0) {
+        for (int i = 0; i < kStages; ++i) mbar_init(bar0 + 8 * i, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+
+    // Producer step (lane 0): tile k of this warp into slot k % kStages.
+    auto issue = [&](int k) {
+        const int ti = tile0 + warp + k * kDecodeWarps;
+        const int tok = ti * kTileTokens;
+        const int j = tok / sh.bt;
+        int blk = trow[j];
+        if (blk < 0 || blk >= sh.num_blocks) {
+            atomicOr(a.err, kErrBadBlock);
+            blk = 0;
+        }
+        const int rowk = ((blk * sh.L + l) * 2 * sh.Hkv + g) * sh.bt + (tok - j * sh.bt);
+        const int rowv = rowk + chunk_rows;
+        const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
+        const uint32_t bar = bar0 + 8 * (k % kStages);
+        mbar_expect_tx(bar, kTileBytes);
+        tma_load_2d(slot, &map, 0, rowk, bar);
+        tma_load_2d(slot + kHalfBytes, &map, 64, rowk, bar);
+        tma_load_2d(slot + 2 * kHalfBytes, &map, 0, rowv, bar);
+        tma_load_2d(slot + 3 * kHalfBytes, &map, 64, rowv, bar);
+    };
+    if (lane == 0)
+        for (int k = 0; k < kStages && k < my_tiles; ++k) issue(k);
+
+    // Q^T fragments (mma B operand): head n = lane/4 of the group, dims
+    // 16*ks + 2*(lane%4) + {0,1} and +8.
+    uint32_t qb[8][2];
+    {
+        const int n = lane >> 2;
+        const bool live = n < G;
+        const uint32_t *qrow = reinterpret_cast<const uint32_t *>(
+            a.q + ((static_cast<int64_t>(li) * a.B + b) * sh.Hq + g * G + (live ? n : 0)) *
+                      kHeadDim);
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+            qb[ks][0] = live ? qrow[ks * 8 + (lane & 3)] : 0u;
+            qb[ks][1] = live ? qrow[ks * 8 + 4 + (lane & 3)] : 0u;
+        }
+    }
+
+    float m0 = -INFINITY, m1 = -INFINITY;   // running max, heads 2(lane%4) and +1
+    float l0 = 0.f, l1 = 0.f;               // this lane's share of the normaliser
+    float o[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+    const float sl = a.scale_log2;
+    int fail_k = -1;
+
+    // ldmatrix lane roles. K (A operand, row-major): row = token.
+    const int krow = (lane & 7) + ((lane >> 3) & 1) * 8;
+    const int khi = lane >> 4;
+    // V (A operand of O^T, loaded transposed): row = token.
+    const int vrow = (lane & 7) + (lane >> 4) * 8;
+    const int vhi = (lane >> 3) & 1;
+
+    for (int k = 0; k < my_tiles; ++k) {
+        const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
+        if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) {
+            fail_k = k;
+            break;
+        }
+        const int ti = tile0 + warp + k * kDecodeWarps;
+        const int tok_base = ti * kTileTokens;
+
+        // S^T = K . Q^T, two accumulators to shorten the mma chain.
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 8; ks += 2) {
+            uint32_t r0, r1, r2, r3;
+            int u = 2 * ks + khi;
+            ldsm_x4(slot + (u >> 3) * kHalfBytes + swz(krow, u & 7), r0, r1, r2, r3);
+            mma_bf16(sa, r0, r1, r2, r3, qb[ks][0], qb[ks][1]);
+            u = 2 * (ks + 1) + khi;
+            ldsm_x4(slot + (u >> 3) * kHalfBytes + swz(krow, u & 7), r0, r1, r2, r3);
+            mma_bf16(sb, r0, r1, r2, r3, qb[ks + 1][0], qb[ks + 1][1]);
+        }
+        const bool v0 = tok_base + (lane >> 2) < T;
+        const bool v1 = tok_base + (lane >> 2) + 8 < T;
+        const float x0 = v0 ? (sa[0] + sb[0]) * sl : -INFINITY;
+        const float x1 = v0 ? (sa[1] + sb[1]) * sl : -INFINITY;
+        const float x2 = v1 ? (sa[2] + sb[2]) * sl : -INFINITY;
+        const float x3 = v1 ? (sa[3] + sb[3]) * sl : -INFINITY;
+        float mx0 = fmaxf(x0, x2), mx1 = fmaxf(x1, x3);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+        }
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+        m0 = mn0;
+        m1 = mn1;
+        float q0, q1, q2, q3;   // P rounded to bf16, as the PV product sees it
+        const uint32_t p01 = pack_bf16(ex2(x0 - mn0), ex2(x1 - mn1), q0, q1);
+        const uint32_t p23 = pack_bf16(ex2(x2 - mn0), ex2(x3 - mn1), q2, q3);
+        l0 = l0 * al0 + q0 + q2;
+        l1 = l1 * al1 + q1 + q3;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            o[i][0] *= al0;
+            o[i][1] *= al1;
+            o[i][2] *= al0;
+            o[i][3] *= al1;
+        }
+        const uint32_t pb0 = movmatrix_t(p01);   // P^T tokens 0-7  -> B fragment
+        const uint32_t pb1 = movmatrix_t(p23);   // P^T tokens 8-15
+
+        const uint32_t vslot = slot + 2 * kHalfBytes;
+        if (tok_base + kTileTokens > T) {
+            // Last, partial tile: slots past T may hold anything (NaN);
+            // P is 0 there but 0 * NaN is not, so clear those V rows.
+            const int first_bad = T - tok_base;
+            const int units = (kTileTokens - first_bad) * 16;
+            uint8_t *vp = ring + (k % kStages) * kTileBytes + 2 * kHalfBytes;
+            for (int u = lane; u < units; u += 32) {
+                const int r = first_bad + (u >> 4);
+                const int h = (u >> 3) & 1;
+                *reinterpret_cast<uint4 *>(vp + h * kHalfBytes + r * 128 + (u & 7) * 16) =
+                    make_uint4(0u, 0u, 0u, 0u);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            uint32_t r0, r1, r2, r3;
+            const int u = 2 * i + vhi;
+            ldsm_x4_t(vslot + (u >> 3) * kHalfBytes + swz(vrow, u & 7), r0, r1, r2, r3);
+            mma_bf16(o[i], r0, r1, r2, r3, pb0, pb1);
+        }
+        __syncwarp();
+        if (lane == 0 && k + kStages < my_tiles) issue(k + kStages);
+    }
+
+    if (fail_k >= 0) {
+        if (lane == 0) atomicOr(a.err, kErrTimeout);
+        // Tiles fail_k .. fail_k+kStages-1 were issued and not consumed: wait
+        // (again bounded) for them so no copy lands after the CTA exits.
+        for (int k = fail_k; k < fail_k + kStages && k < my_tiles; ++k)
+            mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1);
+    }
+
+    // Normaliser: reduce the per-lane shares over the 8 lanes of a column.
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+    }
+
+    // Warp state -> own ring (all of its loads have completed).
+    constexpr int kOStride = kHeadDim + 4;   // floats per head row (bank skew)
+    float *ws = reinterpret_cast<float *>(ring);
+    float *wm = ws + kMaxGroup * kOStride;   // m[8], l[8]
+    {
+        const int h0 = 2 * (lane & 3);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int d = 16 * i + (lane >> 2);
+            ws[h0 * kOStride + d] = o[i][0];
+            ws[(h0 + 1) * kOStride + d] = o[i][1];
+            ws[h0 * kOStride + d + 8] = o[i][2];
+            ws[(h0 + 1) * kOStride + d + 8] = o[i][3];
+        }
+        if (lane < 4) {
+            wm[h0] = m0;
+            wm[h0 + 1] = m1;
+            wm[8 + h0] = l0;
+            wm[8 + h0 + 1] = l1;
+        }
+    }
+    __syncthreads();
+
+    // Merge warps in fixed order; thread handles (head, 8 dims).
+    const int64_t row_base = static_cast<int64_t>(lb) * sh.Hq + g * G;
+    for (int e = threadIdx.x; e < G * (kHeadDim / 8); e += blockDim.x) {
+        const int h = e / (kHeadDim / 8);
+        const int d0 = (e % (kHeadDim / 8)) * 8;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kDecodeWarps; ++w) {
+            const float *wmw =
+                reinterpret_cast<const float *>(smem + w * kStages * kTileBytes) +
+                kMaxGroup * kOStride;
+            M = fmaxf(M, wmw[h]);
+        }
+        float lsum = 0.f, acc[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+#pragma unroll
+        for (int w = 0; w < kDecodeWarps; ++w) {
+            const float *wsw = reinterpret_cast<const float *>(smem + w * kStages * kTileBytes);
+            const float *wmw = wsw + kMaxGroup * kOStride;
+            const float sc = ex2(wmw[h] - M);
+            lsum += sc * wmw[8 + h];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) acc[c] += sc * wsw[h * kOStride + d0 + c];
+        }
+        if (nsplit == 1) {
+            const float inv = 1.f / lsum;
+            float4 *dst = reinterpret_cast<float4 *>(a.out + (row_base + h) * kHeadDim + d0);
+            dst[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+            dst[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+        } else {
+            const int64_t prow = (row_base + h) * a.max_splits + split;
+            float4 *dst = reinterpret_cast<float4 *>(a.part_o + prow * kHeadDim + d0);
+            dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+            dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+            if (d0 == 0) {
+                a.part_ml[prow * 2] = M;
+                a.part_ml[prow * 2 + 1] = lsum;
+            }
+        }
+    }
+}
+
+// K2: one warp per (layer-batch row, q-head); lane owns 4 dims. Splits are
+// merged sequentially in index order, so the sum order is fixed.
+__global__ void __launch_bounds__(256) decode_combine_kernel(const DecodeArgs a) {
+    const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t rows = static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq;
+    if (wid >= rows) return;
+    const int lb = static_cast<int>(wid / a.s.Hq);
+    const int b = lb % a.B;
+    const int T = a.seq_lens[b];
+    if (T < 1 || T > a.max_blocks * a.s.bt) return;
+    const int ns = num_splits(T);
+    if (ns <= 1) return;   // written by the split kernel
+    const int64_t base = wid * a.max_splits;
+    float M = -INFINITY;
+    for (int s = lane; s < ns; s += 32) M = fmaxf(M, a.part_ml[(base + s) * 2]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float lsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 *po = reinterpret_cast<const float4 *>(a.part_o + base * kHeadDim) + lane;
+    for (int s = 0; s < ns; ++s) {
+        const float w = ex2(a.part_ml[(base + s) * 2] - M);
+        lsum += w * a.part_ml[(base + s) * 2 + 1];
+        const float4 v = po[s * (kHeadDim / 4)];
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+    }
+    const float inv = 1.f / lsum;
+    reinterpret_cast<float4 *>(a.out + wid * kHeadDim)[lane] =
+        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+}
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// K3 / K4: one warp per (layer, K|V, kv-head, block) run of the token range.
+// Both sides of a run are contiguous rows of 256 B; a warp moves it with
+// 16-byte loads, eight in flight per lane. Items are ordered run-major so
+// that consecutive warps walk the image sequentially.
+template <bool kPack>
+__global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
+    const Shape sh = a.s;
+    const int runs = sh.L * 2 * sh.Hkv;
+    const int j0 = a.t_begin / sh.bt;
+    const int j1 = (a.t_end + sh.bt - 1) / sh.bt;
+    const int nj = j1 - j0;
+    const int items = runs * nj;
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int it = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; it < items; it += nwarps) {
+        const int c = it / nj;
+        const int j = j0 + (it - c * nj);
+        const int blk = a.table[j];
+        if (blk < 0 || blk >= sh.num_blocks) {
+            if (lane == 0) atomicOr(a.err, kErrBadBlock);
+            continue;
+        }
+        const int t_lo = max(a.t_begin, j * sh.bt);
+        const int t_hi = min(a.t_end, (j + 1) * sh.bt);
+        uint8_t *hp = a.hot + ((static_cast<int64_t>(blk) * runs + c) * sh.bt + (t_lo - j * sh.bt)) *
+                                  kRowBytes;
+        uint8_t *ip = a.img + (static_cast<int64_t>(c) * a.T_cap + t_lo) * kRowBytes;
+        const uint4 *src = reinterpret_cast<const uint4 *>(kPack ? hp : ip);
+        uint4 *dst = reinterpret_cast<uint4 *>(kPack ? ip : hp);
+        const int units = (t_hi - t_lo) * (kRowBytes / 16);
+        for (int u0 = 0; u0 < units; u0 += 32 * 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < units) v[k] = ld_stream(src + u);
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < units) dst[u] = v[k];
+            }
+        }
+    }
+}
+
+// K5: one half-warp per (layer, token, K|V, kv-head) row of 256 B.
+__global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
+    const Shape sh = a.s;
+    const int64_t rows = static_cast<int64_t>(sh.L) * a.n * 2 * sh.Hkv;
+    const int sub = threadIdx.x & 15;
+    const int64_t stride = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
+    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 4; r < rows;
+         r += stride) {
+        const int g = static_cast<int>(r % sh.Hkv);
+        const int kv = static_cast<int>((r / sh.Hkv) & 1);
+        const int i = static_cast<int>((r / (2 * sh.Hkv)) % a.n);
+        const int l = static_cast<int>(r / (2LL * sh.Hkv * a.n));
+        const int64_t t = a.pos0 + i;
+        const int blk = a.table[t / sh.bt];
+        if (blk < 0 || blk >= sh.num_blocks) {
+            if (sub == 0) atomicOr(a.err, kErrBadBlock);
+            continue;
+        }
+        const uint8_t *src =
+            (kv ? a.v : a.k) + ((static_cast<int64_t>(l) * a.n + i) * sh.Hkv + g) * kRowBytes;
+        uint8_t *dst = a.hot + ((((static_cast<int64_t>(blk) * sh.L + l) * 2 + kv) * sh.Hkv + g) *
+                                    sh.bt +
+                                t % sh.bt) *
+                                   kRowBytes;
+        reinterpret_cast<uint4 *>(dst)[sub] = reinterpret_cast<const uint4 *>(src)[sub];
+    }
+}
+
+__global__ void table_write_kernel(const __grid_constant__ TableWriteArgs a) {
+    for (int i = threadIdx.x; i < a.n; i += blockDim.x) a.dst[i] = a.vals[i];
+}
+
+__global__ void gather_tables_kernel(const __grid_constant__ GatherArgs a) {
+    const int r = blockIdx.x;
+    if (r >= a.count) return;
+    const int32_t *src = a.arena + static_cast<int64_t>(a.sids[r]) * a.stride;
+    int32_t *dst = a.tables + static_cast<int64_t>(a.row0 + r) * a.max_blocks;
+    const int n = a.nblk[r];
+    for (int e = threadIdx.x; e < a.max_blocks; e += blockDim.x) dst[e] = e < n ? src[e] : -1;
+    if (threadIdx.x == 0) a.seq_lens[a.row0 + r] = a.lens[r];
+}
+
+}  // namespace
+
+bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why) {
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    if (!encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !fn) {
+            *why = "cuTensorMapEncodeTiled entry point unavailable";
+            return false;
+        }
+        encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kRowBytes)};
+    cuuint32_t box[2] = {64, kTileTokens};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, hot_base, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *why = "cuTensorMapEncodeTiled rejected the hot pool";
+        return false;
+    }
+    return true;
+}
+
+cudaError_t prepare_kernels() {
+    return cudaFuncSetAttribute(decode_split_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kDecodeSmem);
+}
+
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st) {
+    // Every session of the batch has T <= max_blocks * bt, so its splits fit.
+    const int splits = max_splits_for(static_cast<int64_t>(a.max_blocks) * a.s.bt);
+    if (splits > a.max_splits) return cudaErrorInvalidValue;
+    dim3 grid(splits, a.s.Hkv, a.nlayers * a.B);
+    decode_split_kernel<<<grid, kDecodeWarps * 32, kDecodeSmem, st>>>(map, a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t warps = static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq;
+    decode_combine_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+static unsigned mig_grid(int64_t items, int num_sms) {
+    int64_t blocks = (items + 7) / 8;
+    const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+    if (blocks > cap) blocks = cap;
+    return static_cast<unsigned>(blocks < 1 ? 1 : blocks);
+}
+
+cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st) {
+    if (a.t_end <= a.t_begin) return cudaSuccess;
+    const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
+    migrate_kernel<false><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st) {
+    if (a.t_end <= a.t_begin) return cudaSuccess;
+    const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
+    migrate_kernel<true><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st) {
+    const int64_t rows = static_cast<int64_t>(a.s.L) * a.n * 2 * a.s.Hkv;
+    int64_t blocks = (rows + 15) / 16;
+    if (blocks > static_cast<int64_t>(num_sms) * 8) blocks = static_cast<int64_t>(num_sms) * 8;
+    append_kernel<<<static_cast<unsigned>(blocks < 1 ? 1 : blocks), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_table_write(const TableWriteArgs &a, cudaStream_t st) {
+    table_write_kernel<<<1, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherArgs &a, cudaStream_t st) {
+    gather_tables_kernel<<<a.count, 128, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace kvt

@@ -1,0 +1,109 @@
+// Internal interface between the pool runtime (pool.cpp) and the kernels
+// (kernels.cu). Not part of the C ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvt {
+
+constexpr int kHeadDim = 128;     // D; one token row of one head is 256 B
+constexpr int kRowBytes = kHeadDim * 2;
+constexpr int kTileTokens = 16;   // tokens per decode tile (one mma M)
+constexpr int kMaxGroup = 8;      // Hq / Hkv handled by one CTA
+
+// Device-side check flags (OR-ed into the pool's error word).
+constexpr int32_t kErrBadBlock = 1;    // block id outside the pool
+constexpr int32_t kErrBadLength = 2;   // seq_len < 1 or past its table row
+constexpr int32_t kErrTimeout = 4;     // an mbarrier wait gave up
+
+// Split-KV plan. A pure function of the session length, so a session's
+// result never depends on batch composition or placement: split s covers
+// tiles [s*split_tiles, (s+1)*split_tiles) of the ceil(T/16) 16-token tiles.
+__host__ __device__ inline int tiles_of(int T) { return (T + kTileTokens - 1) / kTileTokens; }
+__host__ __device__ inline int split_tiles(int T) {
+    int s = (tiles_of(T) + 15) / 16;   // aim at 16 splits per (session, kv-head)
+    return s < 8 ? 8 : (s > 32 ? 32 : s);
+}
+__host__ __device__ inline int num_splits(int T) {
+    int st = split_tiles(T);
+    return (tiles_of(T) + st - 1) / st;
+}
+// Upper bound of num_splits(T) for T <= max_tokens.
+inline int max_splits_for(int64_t max_tokens) {
+    int64_t tiles = (max_tokens + kTileTokens - 1) / kTileTokens;
+    int64_t a = (tiles + 31) / 32;
+    return (int)(a > 16 ? a : 16);
+}
+
+struct Shape {
+    int32_t L, Hq, Hkv, bt;
+    int64_t num_blocks;
+};
+
+struct DecodeArgs {
+    const uint16_t *q;        // [nl][B][Hq][D] bf16
+    const int32_t *tables;    // [B][max_blocks]
+    const int32_t *seq_lens;  // [B]
+    float *out;               // [nl][B][Hq][D]
+    float *part_o;            // [nl*B][Hq][max_splits][D]
+    float *part_ml;           // [nl*B][Hq][max_splits][2]
+    int32_t *err;
+    int32_t B, max_blocks, layer0, nlayers, max_splits;
+    float scale_log2;         // scale * log2(e)
+    Shape s;
+};
+
+struct MigArgs {
+    const int32_t *table;     // session's block-table row (device)
+    uint8_t *hot;
+    uint8_t *img;
+    int64_t T_cap;            // image rows per (layer, K|V, kv-head) run
+    int32_t t_begin, t_end;   // tokens to move
+    int32_t *err;
+    Shape s;
+};
+
+struct AppendArgs {
+    const uint8_t *k, *v;     // [L][n][Hkv][D] bf16
+    const int32_t *table;
+    uint8_t *hot;
+    int64_t pos0;
+    int32_t n;
+    int32_t *err;
+    Shape s;
+};
+
+constexpr int kTableWriteMax = 2048;
+struct TableWriteArgs {
+    int32_t *dst;
+    int32_t n;
+    int32_t vals[kTableWriteMax];
+};
+
+constexpr int kGatherMax = 512;
+struct GatherArgs {
+    const int32_t *arena;     // [max_sessions][stride]
+    int64_t stride;
+    int32_t *tables;          // [B][max_blocks]
+    int32_t *seq_lens;
+    int32_t max_blocks;
+    int32_t count;            // rows written by this launch
+    int32_t row0;             // first batch row of this launch
+    int32_t sids[kGatherMax];
+    int32_t lens[kGatherMax];
+    int32_t nblk[kGatherMax];
+};
+
+// Host launchers (kernels.cu). Each returns the launch's CUDA status.
+bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why);
+cudaError_t prepare_kernels();  // per-device function attributes
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st);
+cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_table_write(const TableWriteArgs &a, cudaStream_t st);
+cudaError_t launch_gather(const GatherArgs &a, cudaStream_t st);
+
+}  // namespace kvt

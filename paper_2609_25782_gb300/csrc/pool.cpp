@@ -1,0 +1,670 @@
+// Pool runtime behind the C ABI of include/kvtier.h.
+//
+// Owns the host metadata of the hot-cold KV hierarchy (Section 3 of the
+// paper): the hot free list and per-session block tables, the cold-arena
+// placement of per-session images, the session states {ACTIVE, PAUSED}, the
+// write-on-evict watermark (cold_valid), and the CUDA events that order
+// migrations against decode. Device work goes to the kernels in kernels.cu.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "../../include/kvtier.h"
+#include "kvt_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const std::string &msg) {
+    g_last_error = msg;
+    return code;
+}
+
+// splitmix64 (Steele, Lea, Flood 2014): state += golden gamma, then mix.
+uint64_t splitmix64(uint64_t &st) {
+    uint64_t z = (st += 0x9E3779B97F4A7C15ULL);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+// Fisher-Yates from the top; draw j = floor(r * (i+1) / 2^64).
+void fisher_yates(std::vector<int32_t> &v, size_t n, uint64_t seed) {
+    uint64_t st = seed;
+    for (size_t i = n; i-- > 1;) {
+        const uint64_t r = splitmix64(st);
+        const size_t j = static_cast<size_t>((static_cast<unsigned __int128>(r) * (i + 1)) >> 64);
+        std::swap(v[i], v[j]);
+    }
+}
+
+struct Session {
+    int32_t state = KV_SESSION_FREE;
+    int64_t T = 0, cap = 0, cold_valid = 0;
+    int64_t img_off = -1, img_bytes = 0;
+    std::vector<int32_t> blocks;
+    cudaEvent_t ready = nullptr;
+    bool ready_recorded = false;
+    cudaEvent_t appended = nullptr;
+    bool appended_recorded = false;
+};
+
+constexpr int kFenceSlots = 64;
+struct Fence {
+    cudaEvent_t ev = nullptr;
+    uint64_t gen = 0;
+};
+
+class DeviceGuard {
+  public:
+    DeviceGuard(int dev, bool active) : active_(active) {
+        if (active_ && cudaGetDevice(&prev_) == cudaSuccess && prev_ != dev) cudaSetDevice(dev);
+        else prev_ = -1;
+    }
+    ~DeviceGuard() {
+        if (active_ && prev_ >= 0) cudaSetDevice(prev_);
+    }
+
+  private:
+    bool active_;
+    int prev_ = -1;
+};
+
+}  // namespace
+
+struct kv_pool {
+    kv_pool_config cfg{};
+    bool host_only = false;
+    int64_t block_bytes = 0, token_bytes = 0;
+    int32_t table_stride = 0;            // max blocks per session
+    int32_t max_splits = 0;
+    int num_sms = 1;
+    kvt::Shape shape{};
+
+    std::vector<int32_t> free_list;      // top = back
+    std::vector<int16_t> block_fence;    // fence slot of the pack that freed it, or -1
+    std::vector<uint64_t> block_fence_gen;
+    std::vector<Session> sessions;
+    std::map<int64_t, int64_t> cold_free;  // offset -> bytes
+    int64_t cold_used = 0;
+
+    int32_t *d_tables = nullptr;
+    float *d_part_o = nullptr;
+    float *d_part_ml = nullptr;
+    int32_t *d_err = nullptr;
+    CUtensorMap tmap{};
+
+    Fence fences[kFenceSlots];
+    int next_fence = 0;
+    uint64_t fence_gen = 0;
+
+    kv_pool_stats stats{};
+    int32_t inject_countdown = 0;
+
+    // Every CUDA call of the pool goes through here: the failure-injection
+    // hook fires first, then (unless the pool is host-logic only) the call.
+    template <typename F>
+    int cuda(const char *what, F &&fn) {
+        if (inject_countdown > 0 && --inject_countdown == 0)
+            return fail(KV_ERR_CUDA, std::string(what) + ": injected CUDA failure");
+        if (host_only) return KV_OK;
+        cudaError_t e = fn();
+        if (e != cudaSuccess)
+            return fail(KV_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+        return KV_OK;
+    }
+
+    Session *session(int32_t sid) {
+        if (sid < 0 || sid >= static_cast<int32_t>(sessions.size())) return nullptr;
+        Session &s = sessions[sid];
+        return s.state == KV_SESSION_FREE ? nullptr : &s;
+    }
+
+    int64_t image_bytes(int64_t cap) const {
+        return (cap * token_bytes + 255) / 256 * 256;
+    }
+
+    bool cold_alloc(int64_t bytes, int64_t *off) {
+        for (auto it = cold_free.begin(); it != cold_free.end(); ++it) {
+            if (it->second >= bytes) {
+                *off = it->first;
+                const int64_t rest = it->second - bytes;
+                const int64_t at = it->first + bytes;
+                cold_free.erase(it);
+                if (rest > 0) cold_free[at] = rest;
+                cold_used += bytes;
+                return true;
+            }
+        }
+        return false;
+    }
+
+    void cold_release(int64_t off, int64_t bytes) {
+        cold_used -= bytes;
+        auto it = cold_free.emplace(off, bytes).first;
+        auto nx = std::next(it);
+        if (nx != cold_free.end() && it->first + it->second == nx->first) {
+            it->second += nx->second;
+            cold_free.erase(nx);
+        }
+        if (it != cold_free.begin()) {
+            auto pv = std::prev(it);
+            if (pv->first + pv->second == it->first) {
+                pv->second += it->second;
+                cold_free.erase(it);
+            }
+        }
+    }
+
+    // Blocks popped for a session: make `st` wait for the packs that freed
+    // them, if those packs may still be running.
+    int wait_fences(const int32_t *blocks, size_t n, cudaStream_t st) {
+        bool need[kFenceSlots] = {};
+        for (size_t i = 0; i < n; ++i) {
+            const int f = block_fence[blocks[i]];
+            if (f >= 0 && fences[f].gen == block_fence_gen[blocks[i]]) need[f] = true;
+        }
+        for (int f = 0; f < kFenceSlots; ++f) {
+            if (!need[f]) continue;
+            int rc = cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, fences[f].ev, 0); });
+            if (rc) return rc;
+        }
+        return KV_OK;
+    }
+
+    void clear_fences(const int32_t *blocks, size_t n) {
+        for (size_t i = 0; i < n; ++i) block_fence[blocks[i]] = -1;
+    }
+
+    // Write entries [from, from+n) of a session's device table row.
+    int write_table(int32_t sid, const int32_t *vals, int64_t from, int64_t n, cudaStream_t st) {
+        for (int64_t i = 0; i < n; i += kvt::kTableWriteMax) {
+            kvt::TableWriteArgs a;
+            a.dst = d_tables + static_cast<int64_t>(sid) * table_stride + from + i;
+            a.n = static_cast<int32_t>(std::min<int64_t>(kvt::kTableWriteMax, n - i));
+            std::memcpy(a.vals, vals + i, sizeof(int32_t) * a.n);
+            int rc = cuda("table write launch", [&] { return kvt::launch_table_write(a, st); });
+            if (rc) return rc;
+        }
+        return KV_OK;
+    }
+
+    kvt::MigArgs mig_args(int32_t sid, const Session &s) const {
+        kvt::MigArgs m;
+        m.table = d_tables + static_cast<int64_t>(sid) * table_stride;
+        m.hot = static_cast<uint8_t *>(cfg.hot_base);
+        m.img = static_cast<uint8_t *>(cfg.cold_base) + s.img_off;
+        m.T_cap = s.cap;
+        m.t_begin = 0;
+        m.t_end = 0;
+        m.err = d_err;
+        m.s = shape;
+        return m;
+    }
+};
+
+extern "C" {
+
+const char *kv_last_error(void) { return g_last_error.c_str(); }
+
+int64_t kv_token_bytes(const kv_pool_config *c) {
+    return c ? static_cast<int64_t>(c->num_layers) * 2 * c->num_kv_heads * c->head_dim * 2 : 0;
+}
+
+int64_t kv_block_bytes(const kv_pool_config *c) {
+    return c ? kv_token_bytes(c) * c->block_tokens : 0;
+}
+
+int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
+    if (!cfg || !out) return fail(KV_ERR_INVALID_ARG, "kv_pool_create: null argument");
+    const kv_pool_config &c = *cfg;
+    if (c.head_dim != kvt::kHeadDim) return fail(KV_ERR_INVALID_ARG, "head_dim must be 128");
+    if (c.block_tokens != 16 && c.block_tokens != 64)
+        return fail(KV_ERR_INVALID_ARG, "block_tokens must be 16 or 64");
+    if (c.num_layers < 1 || c.num_kv_heads < 1 || c.num_kv_heads > 8 || c.num_q_heads < 1 ||
+        c.num_q_heads % c.num_kv_heads != 0 || c.num_q_heads / c.num_kv_heads > kvt::kMaxGroup ||
+        (c.num_q_heads / c.num_kv_heads) & (c.num_q_heads / c.num_kv_heads - 1))
+        return fail(KV_ERR_INVALID_ARG, "need Hkv in 1..8 and Hq/Hkv in {1,2,4,8}");
+    if (c.max_sessions < 1 || c.max_batch < 1 || c.max_context < 1 || c.num_hot_blocks < 1)
+        return fail(KV_ERR_INVALID_ARG, "max_sessions, max_batch, max_context, num_hot_blocks must be >= 1");
+    if (c.num_hot_blocks > INT32_MAX)
+        return fail(KV_ERR_INVALID_ARG, "num_hot_blocks exceeds int32 block ids");
+    const int64_t rows = c.num_hot_blocks * c.num_layers * 2 * c.num_kv_heads * c.block_tokens;
+    if (rows >= (int64_t(1) << 31))
+        return fail(KV_ERR_INVALID_ARG, "hot pool has 2^31 or more 256-byte rows");
+    if (c.max_context > (int64_t(1) << 30)) return fail(KV_ERR_INVALID_ARG, "max_context too large");
+    const bool host_only = (c.flags & KV_POOL_HOST_LOGIC_ONLY) != 0;
+    if (!host_only) {
+        if (!c.hot_base || !c.cold_base) return fail(KV_ERR_INVALID_ARG, "null arena");
+        if ((reinterpret_cast<uintptr_t>(c.hot_base) & 255) ||
+            (reinterpret_cast<uintptr_t>(c.cold_base) & 255))
+            return fail(KV_ERR_INVALID_ARG, "arenas must be 256-byte aligned");
+    }
+    if (c.cold_bytes < 0) return fail(KV_ERR_INVALID_ARG, "cold_bytes < 0");
+
+    kv_pool *p = new kv_pool;
+    p->cfg = c;
+    p->host_only = host_only;
+    p->token_bytes = kv_token_bytes(&c);
+    p->block_bytes = kv_block_bytes(&c);
+    p->table_stride = static_cast<int32_t>((c.max_context + c.block_tokens - 1) / c.block_tokens);
+    p->max_splits = kvt::max_splits_for(static_cast<int64_t>(p->table_stride) * c.block_tokens);
+    p->shape = kvt::Shape{c.num_layers, c.num_q_heads, c.num_kv_heads, c.block_tokens,
+                          c.num_hot_blocks};
+    p->free_list.resize(c.num_hot_blocks);
+    for (int64_t i = 0; i < c.num_hot_blocks; ++i) p->free_list[i] = static_cast<int32_t>(i);
+    fisher_yates(p->free_list, p->free_list.size(), c.alloc_seed);
+    p->block_fence.assign(c.num_hot_blocks, -1);
+    p->block_fence_gen.assign(c.num_hot_blocks, 0);
+    p->sessions.resize(c.max_sessions);
+    if (c.cold_bytes > 0) p->cold_free[0] = c.cold_bytes;
+
+    if (!host_only) {
+        DeviceGuard dg(c.device, true);
+        auto bail = [&](int rc) {
+            kv_pool_destroy(p);
+            return rc;
+        };
+        if (cudaSetDevice(c.device) != cudaSuccess)
+            return bail(fail(KV_ERR_CUDA, "cudaSetDevice failed"));
+        cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, c.device);
+        const int64_t tbl = static_cast<int64_t>(c.max_sessions) * p->table_stride * 4;
+        const int64_t prow = static_cast<int64_t>(c.max_batch) * c.num_q_heads * p->max_splits;
+        int rc = p->cuda("cudaMalloc(tables)", [&] { return cudaMalloc(&p->d_tables, tbl); });
+        if (!rc) rc = p->cuda("cudaMalloc(partials)", [&] {
+            return cudaMalloc(&p->d_part_o, prow * kvt::kHeadDim * sizeof(float));
+        });
+        if (!rc) rc = p->cuda("cudaMalloc(partials)", [&] {
+            return cudaMalloc(&p->d_part_ml, prow * 2 * sizeof(float));
+        });
+        if (!rc) rc = p->cuda("cudaMalloc(err)", [&] { return cudaMalloc(&p->d_err, 4); });
+        if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_err, 0, 4); });
+        if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_tables, 0xFF, tbl); });
+        if (!rc) rc = p->cuda("kernel attributes", [&] { return kvt::prepare_kernels(); });
+        for (int f = 0; !rc && f < kFenceSlots; ++f)
+            rc = p->cuda("cudaEventCreate", [&] {
+                return cudaEventCreateWithFlags(&p->fences[f].ev, cudaEventDisableTiming);
+            });
+        if (rc) return bail(rc);
+        const char *why = nullptr;
+        if (!kvt::encode_hot_tensor_map(&p->tmap, c.hot_base, rows, &why))
+            return bail(fail(KV_ERR_CUDA, why));
+        if (cudaDeviceSynchronize() != cudaSuccess)
+            return bail(fail(KV_ERR_CUDA, "device synchronise after pool set-up failed"));
+    }
+    p->stats.free_blocks = c.num_hot_blocks;
+    *out = p;
+    return KV_OK;
+}
+
+int kv_pool_destroy(kv_pool *p) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    if (!p->host_only) {
+        DeviceGuard dg(p->cfg.device, true);
+        cudaDeviceSynchronize();
+        for (auto &s : p->sessions) {
+            if (s.ready) cudaEventDestroy(s.ready);
+            if (s.appended) cudaEventDestroy(s.appended);
+        }
+        for (auto &f : p->fences)
+            if (f.ev) cudaEventDestroy(f.ev);
+        cudaFree(p->d_tables);
+        cudaFree(p->d_part_o);
+        cudaFree(p->d_part_ml);
+        cudaFree(p->d_err);
+    }
+    delete p;
+    return KV_OK;
+}
+
+static int create_session(kv_pool *p, int64_t max_tokens, int64_t tokens, int32_t state,
+                          int32_t *sid_out) {
+    if (!p || !sid_out) return fail(KV_ERR_INVALID_ARG, "null argument");
+    if (max_tokens < 1 || max_tokens > p->cfg.max_context)
+        return fail(KV_ERR_INVALID_ARG, "max_tokens must be in 1..max_context");
+    if (tokens < 0 || tokens > max_tokens) return fail(KV_ERR_INVALID_ARG, "tokens out of range");
+    int32_t sid = -1;
+    for (int32_t i = 0; i < static_cast<int32_t>(p->sessions.size()); ++i)
+        if (p->sessions[i].state == KV_SESSION_FREE) {
+            sid = i;
+            break;
+        }
+    if (sid < 0) return fail(KV_ERR_INVALID_ARG, "no free session id (max_sessions reached)");
+    const int64_t bytes = p->image_bytes(max_tokens);
+    int64_t off = 0;
+    if (!p->cold_alloc(bytes, &off))
+        return fail(KV_ERR_NO_COLD_SPACE, "cold arena cannot hold the session image");
+    Session &s = p->sessions[sid];
+    s = Session{};
+    s.state = state;
+    s.cap = max_tokens;
+    s.T = tokens;
+    s.cold_valid = tokens;
+    s.img_off = off;
+    s.img_bytes = bytes;
+    p->stats.cold_bytes_used = p->cold_used;
+    *sid_out = sid;
+    return KV_OK;
+}
+
+int session_create(kv_pool *p, int64_t max_tokens, int32_t *sid_out) {
+    return create_session(p, max_tokens, 0, KV_SESSION_ACTIVE, sid_out);
+}
+
+int session_create_paused(kv_pool *p, int64_t max_tokens, int64_t tokens, int32_t *sid_out) {
+    if (tokens < 1) return fail(KV_ERR_INVALID_ARG, "a paused session needs tokens >= 1");
+    return create_session(p, max_tokens, tokens, KV_SESSION_PAUSED, sid_out);
+}
+
+int session_destroy(kv_pool *p, int32_t sid) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    for (int32_t b : s->blocks) p->free_list.push_back(b);
+    p->stats.free_blocks += static_cast<int64_t>(s->blocks.size());
+    p->stats.used_blocks -= static_cast<int64_t>(s->blocks.size());
+    p->cold_release(s->img_off, s->img_bytes);
+    p->stats.cold_bytes_used = p->cold_used;
+    cudaEvent_t ready = s->ready, appended = s->appended;
+    *s = Session{};
+    s->ready = ready;   // events are kept for reuse by the next session in this slot
+    s->appended = appended;
+    return KV_OK;
+}
+
+static int ensure_event(kv_pool *p, cudaEvent_t *ev) {
+    if (*ev || p->host_only) return KV_OK;
+    return p->cuda("cudaEventCreate",
+                   [&] { return cudaEventCreateWithFlags(ev, cudaEventDisableTiming); });
+}
+
+int session_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_t n,
+                   kv_stream_t stream_) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "append to a paused session");
+    if (n < 1) return fail(KV_ERR_INVALID_ARG, "n must be >= 1");
+    if (!p->host_only && (!k || !v)) return fail(KV_ERR_INVALID_ARG, "null k or v");
+    if (s->T + n > s->cap) return fail(KV_ERR_INVALID_ARG, "append past the session capacity");
+    const int bt = p->cfg.block_tokens;
+    const int64_t have = static_cast<int64_t>(s->blocks.size());
+    const int64_t need = (s->T + n + bt - 1) / bt - have;
+    if (need > static_cast<int64_t>(p->free_list.size()))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "hot pool has too few free blocks for the append");
+
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    std::vector<int32_t> fresh(need);
+    for (int64_t i = 0; i < need; ++i) fresh[i] = p->free_list[p->free_list.size() - 1 - i];
+
+    int rc = ensure_event(p, &s->appended);
+    if (!rc && s->ready_recorded)
+        rc = p->cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s->ready, 0); });
+    if (!rc && need > 0) rc = p->wait_fences(fresh.data(), fresh.size(), st);
+    if (!rc && need > 0) rc = p->write_table(sid, fresh.data(), have, need, st);
+    if (!rc) {
+        kvt::AppendArgs a;
+        a.k = static_cast<const uint8_t *>(k);
+        a.v = static_cast<const uint8_t *>(v);
+        a.table = p->d_tables + static_cast<int64_t>(sid) * p->table_stride;
+        a.hot = static_cast<uint8_t *>(p->cfg.hot_base);
+        a.pos0 = s->T;
+        a.n = n;
+        a.err = p->d_err;
+        a.s = p->shape;
+        rc = p->cuda("append launch", [&] { return kvt::launch_append(a, p->num_sms, st); });
+    }
+    if (!rc)
+        rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->appended, st); });
+    if (rc) return rc;   // host state untouched
+
+    p->free_list.resize(p->free_list.size() - need);
+    p->clear_fences(fresh.data(), fresh.size());
+    s->blocks.insert(s->blocks.end(), fresh.begin(), fresh.end());
+    s->T += n;
+    s->appended_recorded = !p->host_only;
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_appended += static_cast<int64_t>(n) * p->token_bytes;
+    p->stats.appends += 1;
+    return KV_OK;
+}
+
+int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
+                     const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
+                     float *out, kv_stream_t stream_) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
+    if (!q || !block_tables || !seq_lens || !out) return fail(KV_ERR_INVALID_ARG, "null pointer");
+    if (layer < -1 || layer >= p->cfg.num_layers) return fail(KV_ERR_INVALID_ARG, "bad layer");
+    const int nl = layer < 0 ? p->cfg.num_layers : 1;
+    if (B < 1 || static_cast<int64_t>(nl) * B > p->cfg.max_batch || nl * B > 65535)
+        return fail(KV_ERR_INVALID_ARG, "B out of range (layers x B must not exceed max_batch)");
+    if (max_blocks < 1 || max_blocks > p->table_stride)
+        return fail(KV_ERR_INVALID_ARG, "max_blocks must be in 1..ceil(max_context/bt)");
+    if (!(scale == scale) || std::isinf(scale)) return fail(KV_ERR_INVALID_ARG, "scale not finite");
+    DeviceGuard dg(p->cfg.device, true);
+    kvt::DecodeArgs a;
+    a.q = static_cast<const uint16_t *>(q);
+    a.tables = block_tables;
+    a.seq_lens = seq_lens;
+    a.out = out;
+    a.part_o = p->d_part_o;
+    a.part_ml = p->d_part_ml;
+    a.err = p->d_err;
+    a.B = B;
+    a.max_blocks = max_blocks;
+    a.layer0 = layer < 0 ? 0 : layer;
+    a.nlayers = nl;
+    a.max_splits = p->max_splits;
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.s = p->shape;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, st); });
+    if (rc) return rc;
+    p->stats.decodes += 1;
+    return KV_OK;
+}
+
+int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "pause of a session that is not active");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+
+    // Fence slot that will mark the freed blocks; its previous pack must be
+    // complete before the slot is re-recorded.
+    const int f = p->next_fence;
+    int rc = KV_OK;
+    if (p->fences[f].gen != 0)
+        rc = p->cuda("cudaEventSynchronize", [&] { return cudaEventSynchronize(p->fences[f].ev); });
+    if (!rc && s->appended_recorded)
+        rc = p->cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s->appended, 0); });
+    if (!rc && s->ready_recorded)
+        rc = p->cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s->ready, 0); });
+    const int64_t t0 = s->cold_valid, t1 = s->T;
+    if (!rc && t1 > t0) {
+        kvt::MigArgs m = p->mig_args(sid, *s);
+        m.t_begin = static_cast<int32_t>(t0);
+        m.t_end = static_cast<int32_t>(t1);
+        rc = p->cuda("pack launch", [&] { return kvt::launch_pack(m, p->num_sms, st); });
+    }
+    if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(p->fences[f].ev, st); });
+    if (rc) return rc;
+
+    p->next_fence = (f + 1) % kFenceSlots;
+    const uint64_t gen = ++p->fence_gen;
+    p->fences[f].gen = gen;
+    for (int32_t b : s->blocks) {
+        p->free_list.push_back(b);
+        p->block_fence[b] = static_cast<int16_t>(f);
+        p->block_fence_gen[b] = gen;
+    }
+    p->stats.free_blocks += static_cast<int64_t>(s->blocks.size());
+    p->stats.used_blocks -= static_cast<int64_t>(s->blocks.size());
+    p->stats.bytes_packed += (t1 - t0) * p->token_bytes;
+    p->stats.pauses += 1;
+    s->blocks.clear();
+    s->cold_valid = t1;
+    s->state = KV_SESSION_PAUSED;
+    s->ready_recorded = false;
+    s->appended_recorded = false;
+    return KV_OK;
+}
+
+int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    if (s->state != KV_SESSION_PAUSED) return fail(KV_ERR_BAD_STATE, "resume of a session that is not paused");
+    const int bt = p->cfg.block_tokens;
+    const int64_t need = (s->T + bt - 1) / bt;
+    if (need > static_cast<int64_t>(p->free_list.size()))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "hot pool has too few free blocks for the resume");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    std::vector<int32_t> fresh(need);
+    for (int64_t i = 0; i < need; ++i) fresh[i] = p->free_list[p->free_list.size() - 1 - i];
+
+    int rc = ensure_event(p, &s->ready);
+    if (!rc) rc = p->wait_fences(fresh.data(), fresh.size(), st);
+    if (!rc) rc = p->write_table(sid, fresh.data(), 0, need, st);
+    if (!rc) {
+        kvt::MigArgs m = p->mig_args(sid, *s);
+        m.t_begin = 0;
+        m.t_end = static_cast<int32_t>(s->T);
+        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->num_sms, st); });
+    }
+    if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
+    if (rc) return rc;
+
+    p->free_list.resize(p->free_list.size() - need);
+    p->clear_fences(fresh.data(), fresh.size());
+    s->blocks = fresh;
+    s->state = KV_SESSION_ACTIVE;
+    s->ready_recorded = !p->host_only;
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_unpacked += s->T * p->token_bytes;
+    p->stats.resumes += 1;
+    return KV_OK;
+}
+
+int session_ready_event(kv_pool *p, int32_t sid, kv_event_t *ev) {
+    if (!p || !ev) return fail(KV_ERR_INVALID_ARG, "null argument");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    *ev = s->ready_recorded ? reinterpret_cast<kv_event_t>(s->ready) : nullptr;
+    return KV_OK;
+}
+
+int session_info(kv_pool *p, int32_t sid, kv_session_info *out) {
+    if (!p || !out) return fail(KV_ERR_INVALID_ARG, "null argument");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    out->state = s->state;
+    out->num_blocks = static_cast<int32_t>(s->blocks.size());
+    out->tokens = s->T;
+    out->capacity = s->cap;
+    out->cold_valid = s->cold_valid;
+    out->image = p->host_only ? nullptr : static_cast<uint8_t *>(p->cfg.cold_base) + s->img_off;
+    return KV_OK;
+}
+
+int session_block_table(kv_pool *p, int32_t sid, int32_t *host_row, int32_t cap, int32_t *nblocks) {
+    if (!p || !nblocks || (cap > 0 && !host_row)) return fail(KV_ERR_INVALID_ARG, "null argument");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    *nblocks = static_cast<int32_t>(s->blocks.size());
+    const int32_t n = std::min<int32_t>(cap, *nblocks);
+    if (n > 0) std::memcpy(host_row, s->blocks.data(), sizeof(int32_t) * n);
+    return KV_OK;
+}
+
+int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
+                         int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream_) {
+    if (!p || !sids || B < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "batch tables on a host-logic-only pool");
+    if (!block_tables || !seq_lens || max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
+    for (int32_t i = 0; i < B; ++i) {
+        Session *s = p->session(sids[i]);
+        if (!s) return fail(KV_ERR_INVALID_ARG, "no such session in batch");
+        if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "paused session in batch");
+        if (s->T < 1) return fail(KV_ERR_INVALID_ARG, "empty session in batch");
+        if (static_cast<int64_t>(s->blocks.size()) > max_blocks)
+            return fail(KV_ERR_INVALID_ARG, "max_blocks shorter than a session's table");
+    }
+    DeviceGuard dg(p->cfg.device, true);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    for (int32_t r0 = 0; r0 < B; r0 += kvt::kGatherMax) {
+        kvt::GatherArgs a;
+        a.arena = p->d_tables;
+        a.stride = p->table_stride;
+        a.tables = block_tables;
+        a.seq_lens = seq_lens;
+        a.max_blocks = max_blocks;
+        a.row0 = r0;
+        a.count = std::min(B - r0, kvt::kGatherMax);
+        for (int32_t i = 0; i < a.count; ++i) {
+            const Session &s = p->sessions[sids[r0 + i]];
+            a.sids[i] = sids[r0 + i];
+            a.lens[i] = static_cast<int32_t>(s.T);
+            a.nblk[i] = static_cast<int32_t>(s.blocks.size());
+        }
+        int rc = p->cuda("gather launch", [&] { return kvt::launch_gather(a, st); });
+        if (rc) return rc;
+    }
+    return KV_OK;
+}
+
+int kv_pool_shuffle_free(kv_pool *p, uint64_t seed) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    fisher_yates(p->free_list, p->free_list.size(), seed);
+    return KV_OK;
+}
+
+int kv_pool_free_list(kv_pool *p, int32_t *host_out, int64_t cap, int64_t *n) {
+    if (!p || !n || (cap > 0 && !host_out)) return fail(KV_ERR_INVALID_ARG, "null argument");
+    *n = static_cast<int64_t>(p->free_list.size());
+    const int64_t m = std::min<int64_t>(cap, *n);
+    if (m > 0) std::memcpy(host_out, p->free_list.data(), sizeof(int32_t) * m);
+    return KV_OK;
+}
+
+int kv_pool_get_stats(kv_pool *p, kv_pool_stats *out) {
+    if (!p || !out) return fail(KV_ERR_INVALID_ARG, "null argument");
+    *out = p->stats;
+    out->cold_bytes_used = p->cold_used;
+    return KV_OK;
+}
+
+int kv_pool_check_device(kv_pool *p, int32_t *flags) {
+    if (!p || !flags) return fail(KV_ERR_INVALID_ARG, "null argument");
+    *flags = 0;
+    if (p->host_only) return KV_OK;
+    DeviceGuard dg(p->cfg.device, true);
+    int rc = p->cuda("cudaDeviceSynchronize", [&] { return cudaDeviceSynchronize(); });
+    if (!rc) rc = p->cuda("cudaMemcpy", [&] {
+        return cudaMemcpy(flags, p->d_err, 4, cudaMemcpyDeviceToHost);
+    });
+    if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_err, 0, 4); });
+    if (rc) return rc;
+    if (*flags) return fail(KV_ERR_DEVICE_CHECK, "a kernel bounds check fired (flags " + std::to_string(*flags) + ")");
+    return KV_OK;
+}
+
+int kv_pool_inject_cuda_failure(kv_pool *p, int32_t n) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    p->inject_countdown = n > 0 ? n : 0;
+    return KV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,310 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle.
+
+Decode attention must satisfy |gpu - oracle| <= 1e-2 * max(1, |oracle|)
+elementwise; migrated bytes and block tables must be bit-exact; a session's
+decode output must be bit-identical before and after a pause/resume round
+trip, across batch compositions and across physical placements.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+
+
+@pytest.fixture(scope="module")
+def pkg(cuda_dev):
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_25782_gb300 as P
+    return P
+
+
+def scaled_err(got, ref):
+    return np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref))) if ref.size else 0.0
+
+
+def direct_case(P, lens, L=2, Hq=32, Hkv=4, bt=16, seed=0, spare=7, k_scale=1.0, max_batch=None):
+    """Pool whose hot blocks are filled directly by the input generator at a
+    seeded random placement (decode tested on its own)."""
+    dev = torch.device("cuda:0")
+    nb = int(sum(-(-t // bt) for t in lens)) + spare
+    max_ctx = max(max(lens), bt)
+    pool = P.Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, num_q_heads=Hq,
+                  num_kv_heads=Hkv, block_tokens=bt, max_sessions=4,
+                  max_batch=max_batch or L * len(lens), max_context=max_ctx)
+    tables = synth.random_block_tables(seed, lens, bt, nb)
+    sess = list(range(len(lens)))
+    synth.fill_hot_pool_torch(pool.hot, seed, sess, lens, tables, L, Hkv, 128, bt, k_scale)
+    q = synth.queries_torch(seed, sess, range(L), Hq, 128, dev)
+    return pool, sess, tables, q
+
+
+def gpu_decode(pool, layer, q, tables, lens):
+    dev = torch.device("cuda:0")
+    t = torch.as_tensor(tables, device=dev)
+    s = torch.as_tensor(np.asarray(lens, dtype=np.int32), device=dev)
+    B = len(lens)
+    shape = (pool.L if layer < 0 else 1, B, pool.Hq, 128)
+    out = torch.full(shape, float("nan"), dtype=torch.float32, device=dev)
+    qq = q if layer < 0 else q[layer:layer + 1]
+    pool.decode_attention(layer, qq.contiguous(), t, s, B, t.shape[1],
+                          getattr(pool, "_scale", 1 / math.sqrt(128)), out)
+    torch.cuda.synchronize()
+    return out.cpu().double().numpy()
+
+
+def host_hot(pool, seed, sess, lens, tables, k_scale=1.0):
+    return synth.hot_pool_np(seed, sess, lens, tables, pool.num_hot_blocks, pool.L, pool.Hkv,
+                             128, pool.bt, k_scale)
+
+
+LENGTHS = [1, 2, 15, 16, 17, 31, 33, 63, 64, 65, 127, 128, 129, 255, 511, 512, 513, 1000,
+           1793, 2049, 4097, 8191, 8193]
+
+
+def test_decode_many_lengths_all_and_per_layer(pkg):
+    lens = LENGTHS
+    pool, sess, tables, q = direct_case(pkg, lens, L=2, seed=1)
+    ref = oracle.paged_decode(host_hot(pool, 1, sess, lens, tables), q.cpu().view(torch.int16)
+                              .numpy().view(np.uint16), tables, lens, 1 / math.sqrt(128), 32)
+    got_all = gpu_decode(pool, -1, q, tables, lens)
+    assert scaled_err(got_all, ref) <= TOL
+    for l in range(2):
+        got = gpu_decode(pool, l, q, tables, lens)
+        assert np.array_equal(got[0], got_all[l])   # one launch per layer == all layers
+    assert pool.check_device() == 0
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(32, 4), (16, 4), (8, 4), (4, 4), (8, 8), (8, 1)])
+def test_decode_group_sizes(pkg, Hq, Hkv):
+    lens = [5, 77, 300, 1500]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, Hq=Hq, Hkv=Hkv, seed=2)
+    hot = synth.hot_pool_np(2, sess, lens, tables, pool.num_hot_blocks, 1, Hkv, 128, 16)
+    ref = oracle.paged_decode(hot, q.cpu().view(torch.int16).numpy().view(np.uint16), tables,
+                              lens, 1 / math.sqrt(128), Hq)
+    assert scaled_err(gpu_decode(pool, -1, q, tables, lens), ref) <= TOL
+
+
+def test_decode_block_64(pkg):
+    lens = [1, 63, 64, 65, 700, 3001]
+    pool, sess, tables, q = direct_case(pkg, lens, L=2, bt=64, seed=3)
+    ref = oracle.paged_decode(host_hot(pool, 3, sess, lens, tables),
+                              q.cpu().view(torch.int16).numpy().view(np.uint16), tables, lens,
+                              1 / math.sqrt(128), 32)
+    assert scaled_err(gpu_decode(pool, -1, q, tables, lens), ref) <= TOL
+
+
+@pytest.mark.parametrize("k_scale,scale", [(1 / math.sqrt(128), 1.0), (1.0, 1 / math.sqrt(128)),
+                                           (1.0, 0.5)])
+def test_decode_scale_readings(pkg, k_scale, scale):
+    lens = [700, 1234]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=4, k_scale=k_scale)
+    pool._scale = scale
+    hot = host_hot(pool, 4, sess, lens, tables, k_scale)
+    ref = oracle.paged_decode(hot, q.cpu().view(torch.int16).numpy().view(np.uint16), tables,
+                              lens, scale, 32)
+    assert scaled_err(gpu_decode(pool, -1, q, tables, lens), ref) <= TOL
+
+
+def test_decode_independent_of_batch_and_placement(pkg):
+    lens = [900, 33, 4100]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=5, spare=300)
+    full = gpu_decode(pool, 0, q, tables, lens)
+    # alone, and in another batch order
+    alone = gpu_decode(pool, 0, q[:, 2:3], tables[2:3], lens[2:3])
+    assert np.array_equal(alone[0, 0], full[0, 2])
+    order = [2, 0, 1]
+    perm = gpu_decode(pool, 0, q[:, order], tables[order], [lens[i] for i in order])
+    for i, o in enumerate(order):
+        assert np.array_equal(perm[0, i], full[0, o])
+    # move every block of session 0 to fresh physical blocks
+    hv = pool.hot_view()
+    used = set(tables[tables >= 0].tolist())
+    free = [b for b in range(pool.num_hot_blocks) if b not in used]
+    n0 = -(-lens[0] // 16)
+    t2 = tables.copy()
+    t2[0, :n0] = free[:n0]
+    src = torch.as_tensor(tables[0, :n0].astype(np.int64), device=hv.device)
+    dst = torch.as_tensor(np.asarray(free[:n0], dtype=np.int64), device=hv.device)
+    hv[dst] = hv[src]
+    moved = gpu_decode(pool, 0, q, t2, lens)
+    assert np.array_equal(moved, full)
+
+
+def test_nan_tail_slots_do_not_leak(pkg):
+    lens = [17, 100, 529]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=6)
+    hv = pool.hot_view()
+    for b, T in enumerate(lens):         # poison every slot past T, K and V
+        j = (T - 1) // 16
+        hv[int(tables[b, j]), :, :, :, T % 16 or 16:, :] = float("nan")
+    got = gpu_decode(pool, 0, q, tables, lens)
+    assert np.all(np.isfinite(got))
+    ref = oracle.paged_decode(host_hot(pool, 6, sess, lens, tables),
+                              q.cpu().view(torch.int16).numpy().view(np.uint16), tables, lens,
+                              1 / math.sqrt(128), 32)
+    assert scaled_err(got, ref) <= TOL
+
+
+def test_device_check_flags(pkg):
+    lens = [40]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=7)
+    bad = tables.copy()
+    bad[0, 1] = pool.num_hot_blocks + 3          # outside the pool: flagged, not read
+    gpu_decode(pool, 0, q, bad, lens)
+    assert pool.check_device() & 1
+    gpu_decode(pool, 0, q, tables, [tables.shape[1] * 16 + 1])   # longer than its table row
+    assert pool.check_device() & 2
+    gpu_decode(pool, 0, q, tables, lens)
+    assert pool.check_device() == 0
+
+
+# ------------------------------------------------------------ migration
+
+def np_bits(t):
+    return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def test_resume_pack_append_bit_exact(pkg):
+    """resume-unpack, append and pause-pack against the oracle's copies, and
+    the block tables against the oracle's free-list contract."""
+    dev = torch.device("cuda:0")
+    L, Hkv, bt, seed, NB = 3, 4, 16, 9, 120
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=NB, cold_bytes=1 << 26, max_sessions=4,
+                    max_batch=8, max_context=1024, alloc_seed=21)
+    ref_fl = oracle.FreeList(NB, 21)
+    hot_ref = np.zeros((NB, L, 2, Hkv, bt, 128), dtype=np.uint16)
+    T0, cap = 301, 700
+    s = pool.session_create_paused(cap, T0)
+    synth.fill_image_torch(pool.image(s), seed, s, L, Hkv, 128, T0)
+    img_ref = np_bits(pool.image(s))
+    pool.session_resume(s)
+    row = ref_fl.pop(-(-T0 // bt))
+    assert pool.session_block_table(s) == list(row)
+    oracle.unpack(img_ref, T0, row, hot_ref)
+    torch.cuda.synchronize()
+    hot = np_bits(pool.hot_view())
+    for j, p in enumerate(row):
+        n = min(bt, T0 - j * bt)
+        assert np.array_equal(hot[p, :, :, :, :n], hot_ref[p, :, :, :, :n])
+
+    # append 3 chunks crossing block boundaries
+    T = T0
+    for n in (3, 40, 1):
+        k, v = synth.kv_logical_torch(seed + 1, s, range(L), Hkv, 128, T, T + n, dev)
+        kk, vv = k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+        pool.session_append(s, kk, vv)
+        need = -(-(T + n) // bt) - len(row)
+        if need > 0:
+            row = np.concatenate([row, ref_fl.pop(need)])
+        oracle.append(hot_ref, row, T, np_bits(kk), np_bits(vv))
+        T += n
+    assert pool.session_block_table(s) == list(row)
+    torch.cuda.synchronize()
+    hot = np_bits(pool.hot_view())
+    for j, p in enumerate(row):
+        n = min(bt, T - j * bt)
+        assert np.array_equal(hot[p, :, :, :, :n], hot_ref[p, :, :, :, :n])
+
+    # pause packs only [T0, T): the image's first T0 tokens are not rewritten
+    before = pool.stats()["bytes_packed"]
+    img_dev = pool.image(s)
+    img_dev[:, :, :, :T0] = 0        # if pack touched these rows they would change
+    pool.session_pause(s)
+    ref_fl.push(row)
+    exp = np.zeros_like(img_ref)
+    written = oracle.pack(hot_ref, row, T0, T, exp)
+    torch.cuda.synchronize()
+    img = np_bits(pool.image(s))
+    assert np.array_equal(img[:, :, :, T0:T], exp[:, :, :, T0:T])
+    assert not np.any(img[:, :, :, :T0])
+    assert pool.stats()["bytes_packed"] - before == written
+    assert pool.free_list() == list(ref_fl.contents())
+    assert pool.check_device() == 0
+
+
+@pytest.mark.parametrize("T", [1, 16, 17, 1000])
+def test_round_trip_byte_identical(pkg, T):
+    """append -> pause (pack) -> resume (unpack into other blocks): the image
+    equals the appended tokens and the new blocks equal the image."""
+    dev = torch.device("cuda:0")
+    L, bt, NB, Hkv = 2, 16, 200, 4
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=NB, cold_bytes=1 << 26, max_sessions=2,
+                    max_batch=4, max_context=2048, alloc_seed=T)
+    s = pool.session_create(1031)
+    k, v = synth.kv_logical_torch(13, s, range(L), Hkv, 128, 0, T, dev)
+    pool.session_append(s, k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous())
+    old = pool.session_block_table(s)
+    pool.session_pause(s)
+    img = pool.image(s)
+    torch.cuda.synchronize()
+    assert torch.equal(img[:, 0, :, :T].view(torch.int16), k.view(torch.int16))
+    assert torch.equal(img[:, 1, :, :T].view(torch.int16), v.view(torch.int16))
+    pool.shuffle_free(T + 1)
+    pool.session_resume(s)
+    row = pool.session_block_table(s)
+    assert len(row) == len(old)
+    hv = pool.hot_view()
+    blocks = hv[torch.as_tensor(row, device=dev, dtype=torch.int64)]
+    as_img = blocks.permute(1, 2, 3, 0, 4, 5).reshape(L, 2, Hkv, -1, 128)[:, :, :, :T]
+    torch.cuda.synchronize()
+    assert torch.equal(as_img.view(torch.int16), img[:, :, :, :T].view(torch.int16))
+    assert pool.check_device() == 0
+
+
+def test_config1_scenario(pkg):
+    """Tiny single-layer case: 4 sessions (512..2048 tokens, one partial tail)
+    decode; a 5th 1024-token session is packed, its blocks freed, the free
+    list scrambled, and it is resumed into 64 other blocks; the step re-run
+    gives bit-identical outputs for all 5 sessions."""
+    dev = torch.device("cuda:0")
+    L, Hq, Hkv, bt, seed = 1, 32, 4, 16, 0
+    lens = [int(x) for x in synth.session_lengths(seed, 4, 512, 2048, bt)] + [1024]
+    NB = sum(-(-t // bt) for t in lens) + 64 + 32
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=NB, cold_bytes=64 << 20, max_sessions=8,
+                    max_batch=8, max_context=2048, alloc_seed=seed)
+    k_scale = 1 / math.sqrt(128)
+    sids = []
+    for T in lens:
+        s = pool.session_create(2048)
+        k, v = synth.kv_logical_torch(seed, s, range(L), Hkv, 128, 0, T, dev, k_scale)
+        pool.session_append(s, k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous())
+        sids.append(s)
+    q = synth.queries_torch(seed, sids, range(L), Hq, 128, dev)
+    mb = 128
+    tables = torch.empty(len(sids), mb, dtype=torch.int32, device=dev)
+    slens = torch.empty(len(sids), dtype=torch.int32, device=dev)
+
+    def step():
+        pool.batch_tables(sids, tables, mb, slens)
+        out = torch.empty(L, len(sids), Hq, 128, dtype=torch.float32, device=dev)
+        pool.decode_attention(-1, q, tables, slens, len(sids), mb, 1.0, out)
+        torch.cuda.synchronize()
+        return out.clone()
+
+    out1 = step()
+    rows = [pool.session_block_table(s) for s in sids]
+    tab_h = np.full((len(sids), mb), -1, dtype=np.int32)
+    for i, r in enumerate(rows):
+        tab_h[i, :len(r)] = r
+    hot_h = synth.hot_pool_np(seed, sids, lens, tab_h, NB, L, Hkv, 128, bt, k_scale)
+    ref = oracle.paged_decode(hot_h, np_bits(q), tab_h, lens, 1.0, Hq)
+    assert scaled_err(out1.cpu().double().numpy(), ref) <= TOL
+
+    s5 = sids[4]
+    pool.session_pause(s5)
+    pool.shuffle_free(12345)
+    pool.session_resume(s5)
+    new_row = pool.session_block_table(s5)
+    assert len(new_row) == 64 and new_row != rows[4]
+    out2 = step()
+    assert torch.equal(out1, out2)
+    assert pool.check_device() == 0
