@@ -223,6 +223,40 @@ int kv_pool_check_device(kv_pool *pool, int32_t *flags);
  * n <= 0 disarms. */
 int kv_pool_inject_cuda_failure(kv_pool *pool, int32_t n);
 
+/* Fixed size of the device scratch used by decode_attention_noalloc. */
+#define KV_NOALLOC_SCRATCH_BYTES (48ll << 20)
+
+/* decode_attention without any allocation. The paper has no counterpart:
+ * this is a deployment variant of decode_attention.
+ *
+ * Who needs it: callers that cannot let a library allocate device memory,
+ * such as a serving engine that reserves nearly all HBM for its own KV and
+ * weight arenas up front (a library cudaMalloc could then fail, or would
+ * break the engine's memory accounting), or code that cannot accept the
+ * device-wide synchronisation that cudaMalloc/cudaFree may cause while
+ * other streams are running. It needs no pool (creating a pool allocates).
+ *
+ * Same arguments and result as decode_attention, with the pool replaced by
+ * `cfg`, of which only num_layers, num_q_heads, num_kv_heads, head_dim,
+ * block_tokens, num_hot_blocks, hot_base and device are read. The split
+ * partials live in one file-scope device array of KV_NOALLOC_SCRATCH_BYTES
+ * (48 MiB) that every GPU loading the library holds until the process exits.
+ * A call needs layers x B x Hq x S x 520 bytes (+256), S the split bound for
+ * max_blocks * block_tokens tokens (at most 64 up to 32K tokens, 16 up to
+ * 8K); larger requests fail with KV_ERR_INVALID_ARG before any work.
+ * It calls no cudaMalloc, cudaFree or allocating library routine.
+ *
+ * The first call on a device, with that device current, looks up the
+ * array's device address (cudaGetSymbolAddress) and sets the decode
+ * kernel's shared-memory attribute; make that first call before any stream
+ * capture. All calls share the one array: calls whose work overlaps on the
+ * GPU (different streams, or different host threads without ordering) race
+ * and give wrong results; order them on one stream. Kernel bounds checks
+ * keep bad block ids or lengths memory-safe but are not reported here. */
+int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer, const void *q,
+                             const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
+                             int32_t max_blocks, float scale, float *out, kv_stream_t stream);
+
 /* Message of the last error on the calling thread ("" if none). */
 const char *kv_last_error(void);
 

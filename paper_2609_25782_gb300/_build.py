@@ -1,6 +1,6 @@
 """Compile libkvtier.so in-tree with nvcc for sm_103a.
 
-The two translation units (kernels.cu, pool.cpp) compile in parallel and are
+The translation units (kernels.cu, pool.cpp, noalloc.cu) compile in parallel and are
 linked with the static CUDA runtime, so the library needs only the driver at
 run time.
 """
@@ -14,7 +14,7 @@ import sys
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libkvtier.so")
-SOURCES = ["kernels.cu", "pool.cpp"]
+SOURCES = ["kernels.cu", "pool.cpp", "noalloc.cu"]
 HEADERS = ["kvt_internal.h", os.path.join("..", "..", "include", "kvtier.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

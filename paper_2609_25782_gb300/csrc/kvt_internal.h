@@ -106,4 +106,7 @@ cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_table_write(const TableWriteArgs &a, cudaStream_t st);
 cudaError_t launch_gather(const GatherArgs &a, cudaStream_t st);
 
+// Sets the message returned by kv_last_error() on this thread (pool.cpp).
+void set_last_error(const char *msg);
+
 }  // namespace kvt

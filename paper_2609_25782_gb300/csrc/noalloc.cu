@@ -1,0 +1,136 @@
+// decode_attention_noalloc: the decode-attention path for callers that must
+// not allocate device memory (see include/kvtier.h).
+//
+// The split-KV decode keeps per-split partial results (running max, sum and
+// an unnormalised 128-float accumulator per split and query head) between
+// its two kernels. The pool-based entry point keeps them in a workspace the
+// pool allocated when it was created; this entry point keeps them in the
+// file-scope device array below instead, so a call makes no allocation at
+// all. Every GPU that loads the library reserves the array until the
+// process exits.
+#include <mutex>
+
+#include "../../include/kvtier.h"
+#include "kvt_internal.h"
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+// Partials (fp32 accumulators, then (max, sum) pairs), then one flag word.
+static __device__ __align__(256) unsigned char g_decode_scratch[KV_NOALLOC_SCRATCH_BYTES];
+
+struct DeviceScratch {
+    unsigned char *ptr = nullptr;   // device address of g_decode_scratch
+    bool ready = false;
+};
+DeviceScratch g_dev[kMaxDevices];
+std::mutex g_mu;
+
+int fail(int code, const char *msg) {
+    kvt::set_last_error(msg);
+    return code;
+}
+
+// Per-device set-up, run by the first call on each device with that device
+// current: the array's device address (the host-side symbol is only a
+// stand-in) and the decode kernel's shared-memory attribute.
+int setup_device(int dev, unsigned char **ptr) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    DeviceScratch &d = g_dev[dev];
+    if (!d.ready) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || !p)
+            return fail(KV_ERR_CUDA, "decode_attention_noalloc: cudaGetSymbolAddress failed");
+        if (kvt::prepare_kernels() != cudaSuccess)
+            return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel attribute set-up failed");
+        d.ptr = static_cast<unsigned char *>(p);
+        d.ready = true;
+    }
+    *ptr = d.ptr;
+    return KV_OK;
+}
+
+}  // namespace
+
+extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer, const void *q,
+                                        const int32_t *block_tables, const int32_t *seq_lens,
+                                        int32_t B, int32_t max_blocks, float scale, float *out,
+                                        kv_stream_t stream) {
+    if (!cfg || !q || !block_tables || !seq_lens || !out || !cfg->hot_base)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: null pointer");
+    const kv_pool_config &c = *cfg;
+    const int G = c.num_kv_heads > 0 ? c.num_q_heads / c.num_kv_heads : 0;
+    if (c.head_dim != kvt::kHeadDim || (c.block_tokens != 16 && c.block_tokens != 64) ||
+        c.num_kv_heads < 1 || c.num_kv_heads > 8 || c.num_q_heads % c.num_kv_heads != 0 ||
+        G < 1 || G > kvt::kMaxGroup || (G & (G - 1)) || c.num_layers < 1 || c.num_hot_blocks < 1)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: unsupported shape");
+    if (reinterpret_cast<uintptr_t>(c.hot_base) & 255)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: hot arena not 256-byte aligned");
+    const int64_t rows = c.num_hot_blocks * c.num_layers * 2 * c.num_kv_heads * c.block_tokens;
+    if (rows >= (int64_t(1) << 31))
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: hot pool too large");
+    if (layer < -1 || layer >= c.num_layers)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: bad layer");
+    const int nl = layer < 0 ? c.num_layers : 1;
+    if (B < 1 || static_cast<int64_t>(nl) * B > 65535 || max_blocks < 1 || max_blocks > (1 << 26))
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: B or max_blocks out of range");
+    if (!(scale == scale) || scale > 3.0e38f || scale < -3.0e38f)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: scale not finite");
+
+    const int splits = kvt::max_splits_for(static_cast<int64_t>(max_blocks) * c.block_tokens);
+    const int64_t prow = static_cast<int64_t>(nl) * B * c.num_q_heads * splits;
+    const int64_t o_bytes = prow * kvt::kHeadDim * 4;
+    const int64_t ml_bytes = prow * 2 * 4;
+    if (o_bytes + ml_bytes + 256 > KV_NOALLOC_SCRATCH_BYTES)
+        return fail(KV_ERR_INVALID_ARG,
+                    "decode_attention_noalloc: batch needs more scratch than the fixed "
+                    "KV_NOALLOC_SCRATCH_BYTES; use decode_attention with a pool, or fewer "
+                    "sessions / shorter max_blocks per call");
+
+    int prev = -1;
+    if (cudaGetDevice(&prev) != cudaSuccess) return fail(KV_ERR_CUDA, "cudaGetDevice failed");
+    if (c.device < 0 || c.device >= kMaxDevices)
+        return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: bad device ordinal");
+    if (prev != c.device && cudaSetDevice(c.device) != cudaSuccess)
+        return fail(KV_ERR_CUDA, "cudaSetDevice failed");
+    struct Restore {
+        int dev, cur;
+        ~Restore() {
+            if (dev >= 0 && dev != cur) cudaSetDevice(dev);
+        }
+    } restore{prev, c.device};
+
+    unsigned char *scratch = nullptr;
+    int rc = setup_device(c.device, &scratch);
+    if (rc) return rc;
+    CUtensorMap map;
+    const char *why = nullptr;
+    if (!kvt::encode_hot_tensor_map(&map, c.hot_base, rows, &why)) return fail(KV_ERR_CUDA, why);
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int32_t *flag = reinterpret_cast<int32_t *>(scratch + KV_NOALLOC_SCRATCH_BYTES - 256);
+    // The flag word is the only scratch that must start at zero; partials are
+    // written before they are read within the call.
+    if (cudaMemsetAsync(flag, 0, sizeof(int32_t), st) != cudaSuccess)
+        return fail(KV_ERR_CUDA, "decode_attention_noalloc: cudaMemsetAsync failed");
+
+    kvt::DecodeArgs a;
+    a.q = static_cast<const uint16_t *>(q);
+    a.tables = block_tables;
+    a.seq_lens = seq_lens;
+    a.out = out;
+    a.part_o = reinterpret_cast<float *>(scratch);
+    a.part_ml = reinterpret_cast<float *>(scratch + o_bytes);
+    a.err = flag;
+    a.B = B;
+    a.max_blocks = max_blocks;
+    a.layer0 = layer < 0 ? 0 : layer;
+    a.nlayers = nl;
+    a.max_splits = splits;
+    a.scale_log2 = scale * 1.4426950408889634f;
+    a.s = kvt::Shape{c.num_layers, c.num_q_heads, c.num_kv_heads, c.block_tokens, c.num_hot_blocks};
+    if (kvt::launch_decode(map, a, st) != cudaSuccess)
+        return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel launch failed");
+    return KV_OK;
+}

@@ -77,6 +77,8 @@ class DeviceGuard {
 
 }  // namespace
 
+void kvt::set_last_error(const char *msg) { g_last_error = msg; }
+
 struct kv_pool {
     kv_pool_config cfg{};
     bool host_only = false;

@@ -35,8 +35,10 @@ EXPORTS = [
     "decode_attention", "session_pause", "session_resume", "session_ready_event",
     "session_info", "session_block_table", "kv_pool_batch_tables", "kv_pool_shuffle_free",
     "kv_pool_free_list", "kv_pool_get_stats", "kv_pool_check_device",
-    "kv_pool_inject_cuda_failure", "kv_last_error",
+    "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
 ]
+
+KV_NOALLOC_SCRATCH_BYTES = 48 << 20
 
 
 class kv_pool_config(C.Structure):
@@ -97,6 +99,8 @@ def _load():
         "kv_pool_check_device": [p, C.POINTER(i32)],
         "kv_pool_inject_cuda_failure": [p, i32],
         "kv_last_error": [],
+        "decode_attention_noalloc": [C.POINTER(kv_pool_config), i32, p, p, p, i32, i32,
+                                     C.c_float, p, p],
     }
     for name, args in sig.items():
         f = getattr(L, name)
@@ -249,6 +253,15 @@ def kv_pool_check_device(pool: int) -> int:
 
 def kv_pool_inject_cuda_failure(pool: int, n: int) -> None:
     _check(lib.kv_pool_inject_cuda_failure(pool, n), "kv_pool_inject_cuda_failure")
+
+
+def decode_attention_noalloc(cfg: kv_pool_config, layer: int, q, block_tables, seq_lens, B: int,
+                             max_blocks: int, scale: float, out, stream=None) -> None:
+    """decode_attention for callers that cannot allocate: no pool, partials in
+    the library's fixed device scratch (see include/kvtier.h)."""
+    _check(lib.decode_attention_noalloc(C.byref(cfg), layer, _addr(q), _addr(block_tables),
+                                        _addr(seq_lens), B, max_blocks, scale, _addr(out),
+                                        _stream(stream)), "decode_attention_noalloc")
 
 
 def make_config(*, num_layers: int, num_q_heads: int = 32, num_kv_heads: int = 4,
