@@ -69,10 +69,11 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
+        time.sleep(0.5)   # let the sampler start before the timed region
         return self
 
     def __exit__(self, *exc):
@@ -109,20 +110,21 @@ class ClockSampler:
 
 # ---------------------------------------------------------------- workloads
 
-def decode_workload(seed: int, rank: int):
+def decode_workload(args, rank: int):
     import torch
     import synth
     from paper_2609_25782_gb300 import Pool
     dev = torch.device("cuda", torch.cuda.current_device())
-    s = seed + 1000 * rank
-    lens = synth.session_lengths(s, B2, TMIN2, TMAX2, BT)
+    s = args.seed + 1000 * rank
+    nl, B = args.layers, args.batch
+    lens = synth.session_lengths(s, B, args.tmin, args.tmax, BT)
     nb = int(sum(-(-int(t) // BT) for t in lens)) + 64
-    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, max_sessions=B2,
-                max_batch=L * B2, max_context=TMAX2, device=dev.index)
-    tables = synth.random_block_tables(s, lens, BT, nb, max_blocks=TMAX2 // BT)
-    sess = list(range(B2))
-    synth.fill_hot_pool_torch(pool.hot, s, sess, lens, tables, L, HKV, D, BT, chunk_blocks=48)
-    q = synth.queries_torch(s, sess, range(L), HQ, D, dev).contiguous()
+    pool = Pool(num_layers=nl, num_hot_blocks=nb, cold_bytes=256, max_sessions=B,
+                max_batch=nl * B, max_context=args.tmax, device=dev.index)
+    tables = synth.random_block_tables(s, lens, BT, nb, max_blocks=-(-args.tmax // BT))
+    sess = list(range(B))
+    synth.fill_hot_pool_torch(pool.hot, s, sess, lens, tables, nl, HKV, D, BT, chunk_blocks=48)
+    q = synth.queries_torch(s, sess, range(nl), HQ, D, dev).contiguous()
     torch.cuda.synchronize()
     return pool, lens, tables, q
 
@@ -132,7 +134,8 @@ def run_decode(args, ws, rank):
     import torch.distributed as dist
     dev = torch.device("cuda", torch.cuda.current_device())
     t_setup = time.time()
-    pool, lens, tables_h, q = decode_workload(args.seed, rank)
+    pool, lens, tables_h, q = decode_workload(args, rank)
+    L, B2 = args.layers, args.batch
     setup_s = time.time() - t_setup
     tables = torch.as_tensor(tables_h, device=dev)
     lens_d = torch.as_tensor(lens.astype(np.int32), device=dev)
@@ -140,7 +143,7 @@ def run_decode(args, ws, rank):
     out = torch.empty(L, B2, HQ, D, dtype=torch.float32, device=dev)
     scale = 1 / math.sqrt(D)
     stream = torch.cuda.Stream(device=dev)
-    kv_bytes = int(lens.sum()) * TOKEN_BYTES          # per 48-layer step
+    kv_bytes = int(lens.sum()) * L * 2 * HKV * D * 2   # per step (all layers)
     q_bytes = B2 * HQ * D * 2
     out_bytes = B2 * HQ * D * 4
     tab_bytes = int(sum(-(-int(t) // BT) for t in lens)) * 4
@@ -231,9 +234,9 @@ def run_migration(args, rank):
     blocks of a pool with 2x headroom) and the reverse pack."""
     import torch
     import synth
-    from paper_2609_25782_gb300 import Pool, kvtier
+    from paper_2609_25782_gb300 import Pool
     dev = torch.device("cuda", torch.cuda.current_device())
-    n_sess, T = 8, 32768
+    n_sess, T = args.mig_sessions, args.mig_tokens
     nb = 2 * n_sess * (T // BT)
     pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=n_sess * T * TOKEN_BYTES + 4096,
                 max_sessions=2 * n_sess, max_batch=8, max_context=T, alloc_seed=args.seed + rank,
@@ -324,6 +327,183 @@ def run_migration(args, rank):
     }
 
 
+def run_trace(args, rank):
+    """Agentic trace: 48 sessions, N_a = 16, decode on one stream and
+    pack/unpack on another; step p50/p99 from events on the decode stream."""
+    import torch
+    import synth
+    from paper_2609_25782_gb300 import Pool, kvtier
+    from paper_2609_25782_gb300 import trace as tr
+    dev = torch.device("cuda", torch.cuda.current_device())
+    cfg = tr.TraceConfig(seed=args.seed + 1000 * rank, steps=args.trace_steps)
+    trace = tr.generate(cfg)
+    plan = tr.plan(cfg, trace)
+    nb = plan["peak_blocks"] + 256
+    pool = Pool(num_layers=cfg.layers, num_hot_blocks=nb, cold_bytes=plan["cold_bytes"] + 4096,
+                max_sessions=cfg.sessions, max_batch=cfg.active_cap,
+                max_context=plan["max_context"], alloc_seed=cfg.seed, device=dev.index)
+    for i, t in enumerate(trace):
+        sid = pool.session_create_paused(plan["caps"][i], t.t0)
+        synth.fill_image_torch(pool.image(sid), cfg.seed, sid, cfg.layers, cfg.num_kv_heads, D,
+                               t.t0)
+    # appended tokens: slices of one seeded random buffer (values do not
+    # change timing); flat so that any [L][n][Hkv][D] prefix is contiguous
+    per_tok = cfg.layers * cfg.num_kv_heads * D
+    buf_k, buf_v = synth.kv_logical_torch(cfg.seed, 4095, range(cfg.layers), cfg.num_kv_heads, D,
+                                          0, cfg.append_max, dev)
+    flat_k, flat_v = buf_k.reshape(-1), buf_v.reshape(-1)
+
+    def kv_source(sid, t0, t1):
+        n = t1 - t0
+        shape = (cfg.layers, n, cfg.num_kv_heads, D)
+        return flat_k[: n * per_tok].view(shape), flat_v[: n * per_tok].view(shape)
+
+    q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(cfg.layers), HQ, D, dev)
+    out = torch.empty(cfg.layers, cfg.active_cap, HQ, D, dtype=torch.float32, device=dev)
+    max_blocks = -(-plan["max_context"] // cfg.block_tokens)
+    tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=dev)
+    seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=dev)
+    dstream = torch.cuda.Stream(device=dev, priority=-1)
+    mstream = torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize()
+    d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
+                       decode_stream=dstream, mig_stream=mstream, tables=tables,
+                       seq_lens=seq_lens, max_blocks=max_blocks)
+    t0 = time.perf_counter()
+    with torch.cuda.stream(dstream):
+        d.run()
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    flags = pool.check_device()
+    steps_ms = sorted(a.elapsed_time(b) for a, b, _ in d.step_events)
+    mig = {"unpack": [0.0, 0], "pack": [0.0, 0]}
+    for kind, a, b, nbytes in d.mig_events:
+        mig[kind][0] += a.elapsed_time(b)
+        mig[kind][1] += nbytes
+    st = pool.stats()
+    pool.close()
+    del buf_k, buf_v, flat_k, flat_v
+    torch.cuda.empty_cache()
+
+    def pct(p):
+        return steps_ms[min(len(steps_ms) - 1, int(round(p / 100 * (len(steps_ms) - 1))))]
+
+    return {
+        "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
+        "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
+        "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2),
+        "mean_batch": round(sum(b for _, _, b in d.step_events) / max(1, len(d.step_events)), 2),
+        "resumes": st["resumes"], "pauses": st["pauses"],
+        "unpack_gb": round(mig["unpack"][1] / 1e9, 2),
+        "unpack_gbs": round(mig["unpack"][1] / max(1e-9, mig["unpack"][0] * 1e-3) / 1e9, 1),
+        "pack_gb": round(mig["pack"][1] / 1e9, 2),
+        "pack_gbs": round(mig["pack"][1] / max(1e-9, mig["pack"][0] * 1e-3) / 1e9, 1),
+        "decode_kv_gb": round(d.counts["decode_tokens"] * TOKEN_BYTES / 1e9, 1),
+        "hot_read_share": round(d.counts["decode_tokens"] * TOKEN_BYTES /
+                                (d.counts["decode_tokens"] * TOKEN_BYTES + mig["unpack"][1]), 4),
+        "device_flags": flags,
+        "trace": "seeded synthetic: T0 U[2K,24K], bursts Geometric(200), pauses Exp(30 s), "
+                 "turn append LogNormal(median 1536, sigma 1, cap 16K), dt 75 ms/step",
+    }
+
+
+SWEEP_B = (1, 8, 32, 128, 256)
+SWEEP_T = (1024, 4096, 16384, 65536, 131072)
+SWEEP_CAP = 120e9
+
+
+def run_sweep(args):
+    """Roofline-fraction curve: decode over (block size, batch, context) with
+    total KV <= 120 GB, per-layer launches and the all-layers launch; then the
+    resume-unpack sweep over single sessions of 1K..128K tokens."""
+    import torch
+    import synth
+    from paper_2609_25782_gb300 import Pool
+    dev = torch.device("cuda", torch.cuda.current_device())
+    peak, _ = hbm_peak()
+    scale = 1 / math.sqrt(D)
+    points = []
+    for bt in (16, 64):
+        pts = [(B, T) for B in SWEEP_B for T in SWEEP_T if B * T * TOKEN_BYTES <= SWEEP_CAP]
+        max_tok = max(B * T for B, T in pts)
+        nb = max_tok // bt + 64
+        Bmax = max(B for B, _ in pts)
+        # workspace rows: the largest of layers x B x Hq x splits(T) over the points
+        need = max(L * B * HQ * max(16, -(-T // 512)) for B, T in pts)
+        ctx = max(SWEEP_T)
+        pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,
+                    max_sessions=4, max_batch=-(-need // (HQ * max(16, -(-ctx // 512)))),
+                    max_context=ctx, device=dev.index)
+        # values: one synthetic session laid over the whole pool (finite N(0,1))
+        synth.fill_hot_pool_torch(pool.hot, args.seed, [0], [nb * bt], [np.arange(nb)], L, HKV, D,
+                                  bt, chunk_blocks=max(1, 48 * 16 // bt))
+        stream = torch.cuda.Stream(device=dev)
+        for B, T in pts:
+            lens = np.full(B, T, dtype=np.int64)
+            tables = synth.random_block_tables(args.seed + B + T, lens, bt, nb)
+            tab = torch.as_tensor(tables, device=dev)
+            sl = torch.as_tensor(lens.astype(np.int32), device=dev)
+            q = synth.queries_torch(args.seed, range(B), range(L), HQ, D, dev).contiguous()
+            out = torch.empty(L, B, HQ, D, dtype=torch.float32, device=dev)
+            res = {"block_tokens": bt, "B": B, "T": T}
+            for mode in ("per_layer", "all_layers"):
+                def step():
+                    if mode == "all_layers":
+                        pool.decode_attention(-1, q, tab, sl, B, tab.shape[1], scale, out, stream)
+                    else:
+                        for l in range(L):
+                            pool.decode_attention(l, q[l], tab, sl, B, tab.shape[1], scale, out[l],
+                                                  stream)
+                kv = B * T * TOKEN_BYTES
+                reps = max(3, min(50, int(2e11 // kv)))
+                for _ in range(2):
+                    step()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                a.record(stream)
+                for _ in range(reps):
+                    step()
+                b.record(stream)
+                torch.cuda.synchronize()
+                ms = a.elapsed_time(b) / reps
+                gbs = kv / (ms * 1e-3) / 1e9
+                res[mode] = {"ms": round(ms, 4), "kv_gbs": round(gbs, 1), "frac": round(gbs / peak, 3)}
+            points.append(res)
+            del q, out, tab, sl
+        flags = pool.check_device()
+        if flags:
+            raise RuntimeError(f"device check flags {flags} in the sweep")
+        pool.close()
+        del pool
+        torch.cuda.empty_cache()
+    # resume-unpack sweep
+    resume = []
+    Tm = max(SWEEP_T)
+    pool = Pool(num_layers=L, num_hot_blocks=Tm // 16 + 64, cold_bytes=Tm * TOKEN_BYTES * 2 + 4096,
+                max_sessions=len(SWEEP_T) + 1, max_batch=4, max_context=Tm, alloc_seed=args.seed,
+                device=dev.index)
+    stream = torch.cuda.Stream(device=dev)
+    for T in SWEEP_T:
+        s = pool.session_create_paused(T, T)
+        synth.fill_image_torch(pool.image(s), args.seed, s, L, HKV, D, T)
+        ms = []
+        for rep in range(6):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            pool.session_resume(s, stream)
+            b.record(stream)
+            torch.cuda.synchronize()
+            if rep >= 2:
+                ms.append(a.elapsed_time(b))
+            pool.session_pause(s, stream)
+        m = statistics.median(ms)
+        rw = 2 * T * TOKEN_BYTES / (m * 1e-3) / 1e9
+        resume.append({"T": T, "ms": round(m, 4), "gbs_rw": round(rw, 1), "frac": round(rw / peak, 3)})
+        pool.session_destroy(s)
+    pool.close()
+    return {"decode": points, "resume": resume, "peak_gbs": peak}
+
+
 def cpu_baseline(res, seed, budget_s=15.0):
     """The oracle on a bounded sample of the same step: layer 0 (then more
     layers while the budget lasts) of all 32 sessions, its KV read from the
@@ -332,6 +512,7 @@ def cpu_baseline(res, seed, budget_s=15.0):
     import oracle
     import synth
     pool, lens, tables = res["pool"], res["lens"], res["tables"]
+    L = pool.L
     hv = pool.hot_view()
     nblk = [-(-int(t) // BT) for t in lens]
     rows = np.concatenate([tables[b, :n] for b, n in enumerate(nblk)]).astype(np.int64)
@@ -354,7 +535,7 @@ def cpu_baseline(res, seed, budget_s=15.0):
         kv += int(np.sum(lens)) * 2 * HKV * D * 2
     return {"value": round(kv / spent / 1e9, 3), "unit": "GB/s", "cores": oracle.threads(),
             "kind": "oracle",
-            "sample": f"layers 0..{layers - 1} of the 32-session step ({kv / 1e9:.2f} GB of KV), "
+            "sample": f"layers 0..{layers - 1} of the {len(lens)}-session step ({kv / 1e9:.2f} GB of KV), "
                       f"fp64 CPU oracle, {spent:.1f} s"}
 
 
@@ -400,12 +581,25 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-secondary", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only-migration", action="store_true",
+                    help="skip the decode step (profiling the migration kernels)")
+    # workload shape; the defaults are the headline decode configuration
+    ap.add_argument("--layers", type=int, default=L)
+    ap.add_argument("--batch", type=int, default=B2)
+    ap.add_argument("--tmin", type=int, default=TMIN2)
+    ap.add_argument("--tmax", type=int, default=TMAX2)
+    ap.add_argument("--mig-sessions", type=int, default=8)
+    ap.add_argument("--mig-tokens", type=int, default=32768)
+    ap.add_argument("--trace-steps", type=int, default=2000)
+    ap.add_argument("--no-trace", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="print the roofline-fraction sweep (block size x batch x context)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -426,6 +620,16 @@ def main():
     if ws > 1:
         dist.barrier()
 
+    if args.sweep:
+        sw = run_sweep(args)
+        if rank == 0:
+            print(json.dumps({"sweep": sw}))
+        return 0
+    if args.only_migration:
+        sec = run_migration(args, rank)
+        if rank == 0:
+            print(json.dumps({"secondary": sec}))
+        return 0
     res = run_decode(args, ws, rank)
     total_ms = res["total_ms"]
     e2e_ms = res["e2e_ms"]
@@ -445,26 +649,37 @@ def main():
 
     secondary = None
     if not args.no_secondary:
+        keep = res["pool"]
+        res["pool"] = None
         secondary = run_migration(args, rank)
+        res["pool"] = keep
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(res, args.seed + 1000 * rank)
     res["pool"].close()
+    del res["pool"]
+    torch.cuda.empty_cache()
+    if secondary is not None and not args.no_trace:
+        secondary["trace"] = run_trace(args, rank)
+    nl, nbatch = args.layers, args.batch
+    headline = (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2)
+    shape = ("Qwen3-Coder-30B-A3B KV shape (48 layers, Hq 32, Hkv 4, D 128, 16-token blocks), "
+             "32 sessions with contexts U[8K,32K]" if headline else
+             f"{nl} layers (Hq 32, Hkv 4, D 128, 16-token blocks), {nbatch} sessions with contexts "
+             f"U[{args.tmin},{args.tmax}] (reduced profiling case)")
 
     if rank == 0:
         line = {
-            "metric": "decode-attn KV GB/s (48-layer step; resume-unpack GB/s and ms in secondary)",
+            "metric": "decode-attn KV GB/s (per step over all layers; resume-unpack GB/s and ms in secondary)",
             "value": round(value, 1), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
             "config": {
-                "workload": "decode-attention step: Qwen3-Coder-30B-A3B KV shape (48 layers, "
-                            "Hq 32, Hkv 4, D 128, 16-token blocks), 32 sessions with contexts "
-                            "U[8K,32K], random physical blocks",
+                "workload": f"decode-attention step: {shape}, random physical blocks",
                 "tokens": int(np.sum(res["lens"])), "kv_gb_per_step": round(res["kv_bytes"] / 1e9, 2),
-                "launches_per_step": 2 * L, "compute": "bf16 inputs, fp32 softmax/accumulate",
-                "l2": "inputs larger than L2 (KV per layer call >1 GB, per step >60 GB)",
+                "launches_per_step": 2 * nl, "compute": "bf16 inputs, fp32 softmax/accumulate",
+                "l2": f"inputs larger than L2 (KV per layer call {res['kv_bytes'] / nl / 1e9:.2f} GB)",
                 "parallelism": f"replicas x{ws} (sessions sharded, no collective)",
             },
             "e2e": {"value": round(e2e, 1), "unit": "GB/s", "h2d_bytes_per_step": res["h2d"],
@@ -474,7 +689,7 @@ def main():
                          "peak_kind": peak_kind,
                          "kernel": "decode_split_kernel + decode_combine_kernel (one layer call)"},
             "cpu_baseline": cpu,
-            "gpu_launches": 2 * L * args.steps,
+            "gpu_launches": 2 * nl * args.steps,
             "clocks": res["clocks"],
             "secondary": secondary,
         }

@@ -75,7 +75,7 @@ typedef struct kv_pool_config {
     int32_t head_dim;       /* D; must be 128                              */
     int32_t block_tokens;   /* bt; 16 or 64                                */
     int32_t max_sessions;   /* session ids are 0 .. max_sessions-1          */
-    int32_t max_batch;      /* largest B passed to decode_attention         */
+    int32_t max_batch;      /* sizes the decode workspace (see decode_attention) */
     int32_t device;         /* CUDA ordinal holding both arenas             */
     int64_t max_context;    /* longest session in tokens (table width)      */
     int64_t num_hot_blocks; /* blocks in the hot arena                      */
@@ -161,8 +161,11 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  * in the last block are never read into the result (they may hold NaN).
  * The result depends only on the values and seq_lens: not on physical
  * placement, batch composition or timing (bit-identical across a
- * pause/resume round trip). B must not exceed max_batch and max_blocks*bt
- * must not exceed max_context rounded up to a block. */
+ * pause/resume round trip). The pool's decode workspace holds
+ * max_batch x Hq x S(max_context) partial rows, S(t) being the split bound
+ * for t tokens (16 up to 8K tokens, then t/512 rounded up); a call needs
+ * layers x B x Hq x S(max_blocks x bt) rows, else KV_ERR_INVALID_ARG. Calls on
+ * one pool share the workspace: issue them in order on one stream. */
 int decode_attention(kv_pool *pool, int32_t layer, const void *q,
                      const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                      int32_t max_blocks, float scale, float *out, kv_stream_t stream);

@@ -5,7 +5,9 @@
 //                          staged by TMA (cp.async.bulk.tensor, 128-byte
 //                          swizzle) into a per-warp mbarrier ring, and the
 //                          group-by-tile products run on mma.sync bf16.
-//   decode_combine_kernel  log-sum-exp merge of the splits, fixed order.
+//   decode_combine_kernel  log-sum-exp merge of the splits in a fixed order,
+//                          launched as a programmatic dependent of the split
+//                          kernel.
 //   migrate_kernel<false>  data path 2: resume-unpack, cold image -> blocks.
 //   migrate_kernel<true>   data path 4: pause-pack, blocks -> cold image,
 //                          tokens [t0, T) only (write-on-evict, Section 3).
@@ -158,6 +160,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 2)
     const Shape sh = a.s;
     const int G = sh.Hq / sh.Hkv;
 
+    // The combine kernel may be scheduled once every CTA of this grid has
+    // started; it still waits for this grid to finish before reading.
+    asm volatile("griddepcontrol.launch_dependents;");
     const int T = a.seq_lens[b];
     if (T < 1 || T > a.max_blocks * sh.bt) {
         if (split == 0 && g == 0 && threadIdx.x == 0) atomicOr(a.err, kErrBadLength);
@@ -396,39 +401,74 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 2)
     }
 }
 
-// K2: one warp per (layer-batch row, q-head); lane owns 4 dims. Splits are
-// merged sequentially in index order, so the sum order is fixed.
-__global__ void __launch_bounds__(256) decode_combine_kernel(const DecodeArgs a) {
-    const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    const int64_t rows = static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq;
-    if (wid >= rows) return;
-    const int lb = static_cast<int>(wid / a.s.Hq);
+// K2: one CTA (4 warps) per (layer-batch row, q-head) of a multi-split
+// session. Warp w merges the contiguous quarter [w*ns/4, (w+1)*ns/4) of the
+// splits with a running log-sum-exp (split order), then warp 0 merges the
+// four warp states in warp order. The result depends only on the partials
+// and ns. Launched as a programmatic dependent of K1: it waits for K1's
+// completion with griddepcontrol.wait, so its CTAs can already be resident
+// while K1 drains.
+__global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int64_t row = blockIdx.x;                // lb * Hq + h
+    const int lb = static_cast<int>(row / a.s.Hq);
     const int b = lb % a.B;
     const int T = a.seq_lens[b];
     if (T < 1 || T > a.max_blocks * a.s.bt) return;
     const int ns = num_splits(T);
-    if (ns <= 1) return;   // written by the split kernel
-    const int64_t base = wid * a.max_splits;
-    float M = -INFINITY;
-    for (int s = lane; s < ns; s += 32) M = fmaxf(M, a.part_ml[(base + s) * 2]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float lsum = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (ns <= 1) return;                           // written by K1
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t base = row * a.max_splits;
+    const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + base;
     const float4 *po = reinterpret_cast<const float4 *>(a.part_o + base * kHeadDim) + lane;
-    for (int s = 0; s < ns; ++s) {
-        const float w = ex2(a.part_ml[(base + s) * 2] - M);
-        lsum += w * a.part_ml[(base + s) * 2 + 1];
-        const float4 v = po[s * (kHeadDim / 4)];
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+    __shared__ float s_m[kDecodeWarps], s_l[kDecodeWarps];
+    __shared__ float4 s_acc[kDecodeWarps][kHeadDim / 4];
+
+    const int s0 = (warp * ns) / kDecodeWarps;
+    const int s1 = ((warp + 1) * ns) / kDecodeWarps;
+    float m = -INFINITY, lsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+    for (int sp = s0; sp < s1; ++sp) {
+        const float2 v = ml[sp];
+        const float4 o = po[sp * (kHeadDim / 4)];
+        const float mn = fmaxf(m, v.x);
+        const float c = ex2(m - mn);               // rescale what is summed so far
+        const float w = ex2(v.x - mn);
+        m = mn;
+        lsum = lsum * c + w * v.y;
+        acc.x = acc.x * c + w * o.x;
+        acc.y = acc.y * c + w * o.y;
+        acc.z = acc.z * c + w * o.z;
+        acc.w = acc.w * c + w * o.w;
     }
-    const float inv = 1.f / lsum;
-    reinterpret_cast<float4 *>(a.out + wid * kHeadDim)[lane] =
-        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    s_acc[warp][lane] = acc;
+    if (lane == 0) {
+        s_m[warp] = m;
+        s_l[warp] = lsum;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        float M = s_m[0];
+#pragma unroll
+        for (int w = 1; w < kDecodeWarps; ++w) M = fmaxf(M, s_m[w]);
+        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+        float l = 0.f;
+#pragma unroll
+        for (int w = 0; w < kDecodeWarps; ++w) {
+            const float c = ex2(s_m[w] - M);       // an empty quarter has m = -inf: c = 0
+            const float4 x = s_acc[w][lane];
+            r.x += c * x.x;
+            r.y += c * x.y;
+            r.z += c * x.z;
+            r.w += c * x.w;
+            l += c * s_l[w];
+        }
+        const float inv = 1.f / l;
+        reinterpret_cast<float4 *>(a.out + row * kHeadDim)[lane] =
+            make_float4(r.x * inv, r.y * inv, r.z * inv, r.w * inv);
+    }
 }
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
@@ -485,31 +525,35 @@ __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
     }
 }
 
-// K5: one half-warp per (layer, token, K|V, kv-head) row of 256 B.
+// K5: one warp per (layer, token): the token's K and V rows for all kv-heads
+// are 2 x Hkv*256 contiguous bytes in the source; each 256-byte head row goes
+// to its (layer, K|V, head) run of the tail block.
 __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
     const Shape sh = a.s;
-    const int64_t rows = static_cast<int64_t>(sh.L) * a.n * 2 * sh.Hkv;
-    const int sub = threadIdx.x & 15;
-    const int64_t stride = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
-    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 4; r < rows;
-         r += stride) {
-        const int g = static_cast<int>(r % sh.Hkv);
-        const int kv = static_cast<int>((r / sh.Hkv) & 1);
-        const int i = static_cast<int>((r / (2 * sh.Hkv)) % a.n);
-        const int l = static_cast<int>(r / (2LL * sh.Hkv * a.n));
+    const int items = sh.L * a.n;
+    const int lane = threadIdx.x & 31;
+    const int units = sh.Hkv * (kRowBytes / 16);   // 16-byte units per K (or V) token
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int it = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; it < items; it += nwarps) {
+        const int l = it / a.n;
+        const int i = it - l * a.n;
         const int64_t t = a.pos0 + i;
         const int blk = a.table[t / sh.bt];
         if (blk < 0 || blk >= sh.num_blocks) {
-            if (sub == 0) atomicOr(a.err, kErrBadBlock);
+            if (lane == 0) atomicOr(a.err, kErrBadBlock);
             continue;
         }
-        const uint8_t *src =
-            (kv ? a.v : a.k) + ((static_cast<int64_t>(l) * a.n + i) * sh.Hkv + g) * kRowBytes;
-        uint8_t *dst = a.hot + ((((static_cast<int64_t>(blk) * sh.L + l) * 2 + kv) * sh.Hkv + g) *
-                                    sh.bt +
-                                t % sh.bt) *
-                                   kRowBytes;
-        reinterpret_cast<uint4 *>(dst)[sub] = reinterpret_cast<const uint4 *>(src)[sub];
+        const int slot = static_cast<int>(t % sh.bt);
+        const int64_t src_off = static_cast<int64_t>(it) * sh.Hkv * kRowBytes;
+        const int64_t run0 = (static_cast<int64_t>(blk) * sh.L + l) * 2 * sh.Hkv;
+        for (int u = lane; u < 2 * units; u += 32) {
+            const int kv = u >= units;
+            const int uu = u - kv * units;
+            const int g = uu >> 4;                  // 16 units per head row
+            const uint4 v = reinterpret_cast<const uint4 *>((kv ? a.v : a.k) + src_off)[uu];
+            uint8_t *dst = a.hot + (((run0 + kv * sh.Hkv + g) * sh.bt + slot) * kRowBytes);
+            reinterpret_cast<uint4 *>(dst)[uu & 15] = v;
+        }
     }
 }
 
@@ -569,9 +613,17 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStrea
     decode_split_kernel<<<grid, kDecodeWarps * 32, kDecodeSmem, st>>>(map, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const int64_t warps = static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq;
-    decode_combine_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, st>>>(a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
+    cfg.blockDim = dim3(kDecodeWarps * 32);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_combine_kernel, a);
 }
 
 static unsigned mig_grid(int64_t items, int num_sms) {
@@ -596,8 +648,8 @@ cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st) {
 }
 
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st) {
-    const int64_t rows = static_cast<int64_t>(a.s.L) * a.n * 2 * a.s.Hkv;
-    int64_t blocks = (rows + 15) / 16;
+    const int64_t warps = static_cast<int64_t>(a.s.L) * a.n;
+    int64_t blocks = (warps + 7) / 8;
     if (blocks > static_cast<int64_t>(num_sms) * 8) blocks = static_cast<int64_t>(num_sms) * 8;
     append_kernel<<<static_cast<unsigned>(blocks < 1 ? 1 : blocks), 256, 0, st>>>(a);
     return cudaGetLastError();

@@ -84,7 +84,8 @@ struct kv_pool {
     bool host_only = false;
     int64_t block_bytes = 0, token_bytes = 0;
     int32_t table_stride = 0;            // max blocks per session
-    int32_t max_splits = 0;
+    int32_t max_splits = 0;              // split bound for max_context
+    int64_t part_rows = 0;               // decode workspace capacity (partial rows)
     int num_sms = 1;
     kvt::Shape shape{};
 
@@ -277,6 +278,7 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
         cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, c.device);
         const int64_t tbl = static_cast<int64_t>(c.max_sessions) * p->table_stride * 4;
         const int64_t prow = static_cast<int64_t>(c.max_batch) * c.num_q_heads * p->max_splits;
+        p->part_rows = prow;
         int rc = p->cuda("cudaMalloc(tables)", [&] { return cudaMalloc(&p->d_tables, tbl); });
         if (!rc) rc = p->cuda("cudaMalloc(partials)", [&] {
             return cudaMalloc(&p->d_part_o, prow * kvt::kHeadDim * sizeof(float));
@@ -446,10 +448,16 @@ int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *bl
     if (!q || !block_tables || !seq_lens || !out) return fail(KV_ERR_INVALID_ARG, "null pointer");
     if (layer < -1 || layer >= p->cfg.num_layers) return fail(KV_ERR_INVALID_ARG, "bad layer");
     const int nl = layer < 0 ? p->cfg.num_layers : 1;
-    if (B < 1 || static_cast<int64_t>(nl) * B > p->cfg.max_batch || nl * B > 65535)
-        return fail(KV_ERR_INVALID_ARG, "B out of range (layers x B must not exceed max_batch)");
-    if (max_blocks < 1 || max_blocks > p->table_stride)
-        return fail(KV_ERR_INVALID_ARG, "max_blocks must be in 1..ceil(max_context/bt)");
+    if (B < 1 || static_cast<int64_t>(nl) * B > 65535)
+        return fail(KV_ERR_INVALID_ARG, "B out of range");
+    if (max_blocks < 1 || max_blocks > (1 << 26))
+        return fail(KV_ERR_INVALID_ARG, "max_blocks out of range");
+    const int splits = kvt::max_splits_for(static_cast<int64_t>(max_blocks) * p->cfg.block_tokens);
+    const int64_t rows = static_cast<int64_t>(nl) * B * p->cfg.num_q_heads * splits;
+    if (rows > p->part_rows)
+        return fail(KV_ERR_INVALID_ARG,
+                    "decode workspace too small: layers x B x Hq x splits(max_blocks) exceeds "
+                    "max_batch x Hq x splits(max_context)");
     if (!(scale == scale) || std::isinf(scale)) return fail(KV_ERR_INVALID_ARG, "scale not finite");
     DeviceGuard dg(p->cfg.device, true);
     kvt::DecodeArgs a;
@@ -464,7 +472,7 @@ int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *bl
     a.max_blocks = max_blocks;
     a.layer0 = layer < 0 ? 0 : layer;
     a.nlayers = nl;
-    a.max_splits = p->max_splits;
+    a.max_splits = splits;
     a.scale_log2 = scale * 1.4426950408889634f;
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);

@@ -1,0 +1,243 @@
+"""Host trace driver: agentic sessions over the hot/cold KV pool.
+
+Sessions alternate decode bursts with pauses (tool calls, user input); a
+batching scheduler keeps at most N_a sessions decoding and admits a waiting
+session whenever one pauses (the paper's Section 4 methodology). On a pause
+the session's new KV is packed into its cold image and its hot blocks are
+freed (data path 4, write-on-evict); on admission its image is unpacked into
+fresh blocks (data path 2) and the turn's new context is appended (data path
+3). Decode (data path 1) runs on one stream, migrations on another, so
+eviction and resume overlap decode (Section 3, data paths).
+
+The schedule is a pure function of the seeded trace: a session admitted at
+step k first decodes at step k+1 (one step of prefetch), and the decode
+stream waits for its admission event, so a late migration shows up as a
+longer step rather than a different schedule. The same driver runs on a
+host-logic-only pool (no GPU) to size the arenas before the real run.
+
+Every data movement is a C-ABI call into libkvtier.so; this module only
+decides what to call and when.
+"""
+from __future__ import annotations
+
+import heapq
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+from . import kvtier
+
+
+@dataclass
+class TraceConfig:
+    sessions: int = 48
+    t0_min: int = 2048
+    t0_max: int = 24576
+    burst_mean: float = 200.0        # tokens per decode burst (geometric)
+    pause_mean_s: float = 30.0       # seconds (exponential)
+    append_median: float = 1536.0    # tokens per turn (lognormal)
+    append_sigma: float = 1.0        # assumed; only the median is specified
+    append_max: int = 16384          # cap on one turn's appended context
+    active_cap: int = 16             # N_a
+    steps: int = 2000
+    dt_s: float = 0.075              # simulated seconds per decode step (assumed)
+    layers: int = 48
+    num_q_heads: int = 32
+    num_kv_heads: int = 4
+    block_tokens: int = 16
+    seed: int = 0
+
+
+@dataclass
+class SessionTrace:
+    t0: int
+    first_ready_s: float
+    bursts: list = field(default_factory=list)    # tokens per turn
+    pauses: list = field(default_factory=list)    # seconds after each turn
+    appends: list = field(default_factory=list)   # context tokens at each turn start
+
+
+def generate(cfg: TraceConfig, max_turns: int = 64) -> list[SessionTrace]:
+    """Seeded per-session turn sequences (independent arrival phases)."""
+    rng = np.random.Generator(np.random.PCG64(cfg.seed ^ 0x7A3CE))
+    out = []
+    p = 1.0 / cfg.burst_mean
+    for _ in range(cfg.sessions):
+        st = SessionTrace(t0=int(rng.integers(cfg.t0_min, cfg.t0_max + 1)),
+                          first_ready_s=float(rng.uniform(0.0, cfg.pause_mean_s)))
+        st.bursts = [int(x) for x in rng.geometric(p, size=max_turns)]
+        st.pauses = [float(x) for x in rng.exponential(cfg.pause_mean_s, size=max_turns)]
+        app = rng.lognormal(math.log(cfg.append_median), cfg.append_sigma, size=max_turns)
+        st.appends = [int(min(cfg.append_max, max(1, round(x)))) for x in app]
+        out.append(st)
+    return out
+
+
+class TraceDriver:
+    """Runs the schedule against a pool handle.
+
+    gpu=False: host-logic-only pool, no CUDA; records the peak sizes.
+    gpu=True : real pool; `kv_source(sid, t0, t1)` returns device bf16 K and V
+    [L][t1-t0][Hkv][D] for the tokens appended at positions t0..t1-1.
+    """
+
+    def __init__(self, cfg: TraceConfig, pool: int, trace: list[SessionTrace], gpu: bool,
+                 kv_source=None, q=None, out=None, decode_stream=None, mig_stream=None,
+                 tables=None, seq_lens=None, max_blocks: int = 0, on_step=None):
+        self.cfg, self.pool, self.trace, self.gpu = cfg, pool, trace, gpu
+        self.kv_source = kv_source
+        self.q, self.out = q, out
+        self.dstream, self.mstream = decode_stream, mig_stream
+        self.tables, self.seq_lens, self.max_blocks = tables, seq_lens, max_blocks
+        self.on_step = on_step
+        n = cfg.sessions
+        self.sids = list(range(n))           # session i has pool id sids[i]
+        self.turn = [0] * n
+        self.tokens = [t.t0 for t in trace]
+        self.burst_left = [0] * n
+        self.queue = [(t.first_ready_s, i) for i, t in enumerate(trace)]
+        heapq.heapify(self.queue)
+        self.active: list[int] = []          # decoding this step
+        self.joining: list[int] = []         # admitted this step, decode from the next
+        self.retire: list[int] = []
+        self.peak_tokens = list(self.tokens)
+        self.peak_blocks = 0
+        self.counts = {"resumes": 0, "pauses": 0, "appended_tokens": 0, "decode_tokens": 0,
+                       "turn_tokens": 0, "steps": 0}
+        self.step_events = []                # (start, end) per step (gpu)
+        self.mig_events = []                 # (kind, start, end, bytes)
+        self.admit_ev = {}
+        self.last_decode_ev = None
+        if gpu:
+            import torch
+            self._torch = torch
+
+    # ---------------------------------------------------------------- helpers
+    def _event(self):
+        return self._torch.cuda.Event(enable_timing=True)
+
+    def _record_mig(self, kind, fn, nbytes):
+        if not self.gpu:
+            fn()
+            return
+        a, b = self._event(), self._event()
+        a.record(self.mstream)
+        fn()
+        b.record(self.mstream)
+        self.mig_events.append((kind, a, b, nbytes))
+
+    def _append(self, i, n, stream):
+        sid = self.sids[i]
+        t0 = self.tokens[i]
+        if self.gpu:
+            k, v = self.kv_source(sid, t0, t0 + n)
+            kvtier.session_append(self.pool, sid, k, v, n, stream)
+        else:
+            kvtier.session_append(self.pool, sid, None, None, n, None)
+        self.tokens[i] += n
+        self.peak_tokens[i] = max(self.peak_tokens[i], self.tokens[i])
+
+    # ------------------------------------------------------------------- step
+    def step(self, k: int) -> None:
+        cfg = self.cfg
+        now = k * cfg.dt_s
+        tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
+        # 1. sessions whose burst ended last step pause (pack new tokens, free blocks)
+        if self.retire and self.gpu and self.last_decode_ev is not None:
+            self.mstream.wait_event(self.last_decode_ev)
+        for i in self.retire:
+            sid = self.sids[i]
+            info = kvtier.session_info(self.pool, sid)
+            nbytes = (info.tokens - info.cold_valid) * tok_bytes
+            self._record_mig("pack", lambda: kvtier.session_pause(
+                self.pool, sid, self.mstream if self.gpu else None), nbytes)
+            self.active.remove(i)
+            heapq.heappush(self.queue, (now + self.trace[i].pauses[self.turn[i]], i))
+            self.turn[i] += 1
+            self.counts["pauses"] += 1
+        self.retire = []
+        # sessions admitted last step join the batch now
+        self.active.extend(self.joining)
+        self.joining = []
+        # 2. admit ready sessions while below the cap (resume + turn context)
+        while (len(self.active) + len(self.joining) < cfg.active_cap and self.queue
+               and self.queue[0][0] <= now):
+            _, i = heapq.heappop(self.queue)
+            sid = self.sids[i]
+            info = kvtier.session_info(self.pool, sid)
+            self._record_mig("unpack", lambda: kvtier.session_resume(
+                self.pool, sid, self.mstream if self.gpu else None), info.tokens * tok_bytes)
+            n_ctx = self.trace[i].appends[self.turn[i]]
+            self._append(i, n_ctx, self.mstream if self.gpu else None)
+            self.counts["turn_tokens"] += n_ctx
+            self.burst_left[i] = self.trace[i].bursts[self.turn[i]]
+            if self.gpu:
+                ev = self._torch.cuda.Event()
+                ev.record(self.mstream)
+                self.admit_ev[i] = ev
+            self.joining.append(i)
+            self.counts["resumes"] += 1
+        # 3. decode step for the active batch
+        members = sorted(self.active)
+        if members:
+            if self.gpu:
+                start, end = self._event(), self._event()
+                start.record(self.dstream)
+                for i in members:
+                    ev = self.admit_ev.pop(i, None)
+                    if ev is not None:
+                        self.dstream.wait_event(ev)
+            for i in members:                 # this step's token (path 3)
+                self._append(i, 1, self.dstream if self.gpu else None)
+            self.counts["appended_tokens"] += len(members)
+            blocks = sum(-(-self.tokens[i] // cfg.block_tokens) for i in self.active + self.joining)
+            self.peak_blocks = max(self.peak_blocks, blocks)
+            if self.gpu:
+                sids = [self.sids[i] for i in members]
+                B = len(sids)
+                kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
+                                            self.seq_lens, self.dstream)
+                for l in range(cfg.layers):
+                    kvtier.decode_attention(self.pool, l, self.q[l], self.tables, self.seq_lens,
+                                            B, self.max_blocks, 1 / math.sqrt(128), self.out[l],
+                                            self.dstream)
+                end.record(self.dstream)
+                self.last_decode_ev = end
+                self.step_events.append((start, end, B))
+                if self.on_step is not None:
+                    self.on_step(k, members)
+            self.counts["decode_tokens"] += sum(self.tokens[i] for i in members)
+            for i in members:
+                self.burst_left[i] -= 1
+                if self.burst_left[i] <= 0:
+                    self.retire.append(i)
+        self.counts["steps"] += 1
+
+    def run(self, steps: int | None = None) -> None:
+        for k in range(self.cfg.steps if steps is None else steps):
+            self.step(k)
+
+
+def plan(cfg: TraceConfig, trace: list[SessionTrace]) -> dict:
+    """Dry run on a host-logic-only pool: per-session capacity and peak hot
+    blocks needed by the real run (the schedule does not depend on timing)."""
+    tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
+    big = cfg.sessions * (1 << 22) * tok_bytes    # host-logic pool: nothing is allocated
+    c = kvtier.make_config(num_layers=cfg.layers, num_q_heads=cfg.num_q_heads,
+                           num_kv_heads=cfg.num_kv_heads, block_tokens=cfg.block_tokens,
+                           max_sessions=cfg.sessions, max_batch=cfg.active_cap,
+                           max_context=1 << 22, num_hot_blocks=300000,
+                           cold_bytes=big, flags=kvtier.KV_POOL_HOST_LOGIC_ONLY)
+    pool = kvtier.kv_pool_create(c)
+    try:
+        for t in trace:
+            kvtier.session_create_paused(pool, 1 << 22, t.t0)
+        d = TraceDriver(cfg, pool, trace, gpu=False)
+        d.run()
+    finally:
+        kvtier.kv_pool_destroy(pool)
+    caps = [int(x) for x in d.peak_tokens]
+    return {"caps": caps, "peak_blocks": int(d.peak_blocks), "counts": d.counts,
+            "cold_bytes": int(sum(-(-(cap * tok_bytes) // 256) * 256 for cap in caps)),
+            "max_context": int(max(caps))}

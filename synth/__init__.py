@@ -123,6 +123,17 @@ def session_kv_np(seed: int, sess: int, layers, num_kv_heads: int, head_dim: int
     return k, v
 
 
+def token_kv_np(seed: int, sess: int, layer: int, t: int, num_kv_heads: int, head_dim: int,
+                k_scale: float = 1.0):
+    """K and V of one token of one layer: two uint16 arrays [Hkv][D]."""
+    key = key_of(seed, SALT_KV)
+    g = np.arange(num_kv_heads, dtype=np.uint64)[:, None]
+    d = np.arange(head_dim, dtype=np.uint64)[None, :]
+    k = normal_bf16_np(key, kv_index_np(sess, layer, 0, g, t, d), k_scale)
+    v = normal_bf16_np(key, kv_index_np(sess, layer, 1, g, t, d), 1.0)
+    return k, v
+
+
 def queries_np(seed: int, sess_ids, layers, num_q_heads: int, head_dim: int):
     """Q bits [len(layers)][len(sess_ids)][Hq][D] uint16."""
     key = key_of(seed, SALT_Q)

@@ -1,0 +1,227 @@
+"""Parity at the benchmark's full sizes, in the benchmark's launch configuration.
+
+* Decode, 48 layers x 32 sessions x U[8K, 32K] tokens (about 66 GB of KV),
+  one decode_attention call per layer as bench.py issues them. The oracle
+  checks sampled outputs: every layer of two seeded sessions plus one seeded
+  layer of every other session. Its inputs are the generator's values: the
+  device pool is filled by the torch side of the generator (checked against
+  the numpy side on sampled tokens) and the sampled sessions' blocks are
+  copied to the host.
+* Resume burst, 8 x 32K-token images: block tables against the oracle's
+  placement contract, every migrated byte compared on the device, a sampled
+  host re-check through the oracle's unpack, and the reverse pack.
+* Sweep points: 128K-token contexts, 256 sessions, 64-token blocks, and the
+  all-layers launch used for small batches.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+L, HQ, HKV, D = 48, 32, 4, 128
+
+
+@pytest.fixture(scope="module")
+def P(cuda_dev):
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_25782_gb300 as pkg
+    return pkg
+
+
+@pytest.fixture(autouse=True)
+def _release_memory():
+    yield
+    import gc
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+def bits(t):
+    return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def scaled_err(got, ref):
+    return float(np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref))))
+
+
+def host_compact(hot_view, table_row, T, layers, bt):
+    """Host copy of one session's blocks (selected layers), compact table."""
+    nblk = -(-T // bt)
+    idx = torch.as_tensor(np.asarray(table_row[:nblk], dtype=np.int64), device=hot_view.device)
+    blocks = hot_view[idx][:, layers]
+    return bits(blocks), np.arange(nblk, dtype=np.int32)[None, :]
+
+
+def check_generator_sample(hot_view, seed, sid, table_row, T, bt, rng):
+    """The torch fill wrote the numpy generator's values (sampled tokens)."""
+    for t in rng.integers(0, T, size=4):
+        l = int(rng.integers(0, hot_view.shape[1]))
+        k, v = synth.token_kv_np(seed, sid, l, int(t), HKV, D)
+        blk = int(table_row[t // bt])
+        got = bits(hot_view[blk, l, :, :, t % bt])          # [2][Hkv][D]
+        assert np.array_equal(got[0], k) and np.array_equal(got[1], v)
+
+
+def decode_sampled(pool, seed, lens, tables, q, out, layers_for, bt):
+    """Oracle check of out[l][b] for the (session, layers) pairs in layers_for."""
+    hv = pool.hot_view()
+    rng = np.random.default_rng(seed + 99)
+    qh_all = bits(q)
+    worst = 0.0
+    for b, layers in layers_for.items():
+        T = int(lens[b])
+        check_generator_sample(hv, seed, b, tables[b], T, bt, rng)
+        host, tab = host_compact(hv, tables[b], T, layers, bt)
+        qh = np.ascontiguousarray(qh_all[layers][:, b:b + 1])
+        ref = oracle.paged_decode(host, qh, tab, [T], 1 / math.sqrt(D), HQ)
+        got = out[layers][:, b:b + 1].double().cpu().numpy()
+        worst = max(worst, scaled_err(got, ref))
+    return worst
+
+
+def test_decode_full_size_bench_configuration(P, cuda_dev):
+    seed, B, bt = 0, 32, 16
+    lens = synth.session_lengths(seed, B, 8192, 32768, bt)
+    nb = int(sum(-(-int(t) // bt) for t in lens)) + 64
+    pool = P.Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, max_sessions=B,
+                  max_batch=L * B, max_context=32768)
+    tables = synth.random_block_tables(seed, lens, bt, nb, max_blocks=32768 // bt)
+    synth.fill_hot_pool_torch(pool.hot, seed, list(range(B)), lens, tables, L, HKV, D, bt,
+                              chunk_blocks=48)
+    q = synth.queries_torch(seed, range(B), range(L), HQ, D, cuda_dev).contiguous()
+    tab_d = torch.as_tensor(tables, device=cuda_dev)
+    len_d = torch.as_tensor(lens.astype(np.int32), device=cuda_dev)
+    out = torch.full((L, B, HQ, D), float("nan"), dtype=torch.float32, device=cuda_dev)
+    stream = torch.cuda.Stream()
+    for l in range(L):           # the benchmark's launch configuration
+        pool.decode_attention(l, q[l], tab_d, len_d, B, tab_d.shape[1], 1 / math.sqrt(D), out[l],
+                              stream)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    assert torch.isfinite(out).all()
+    rng = np.random.default_rng(7)
+    full = [int(x) for x in rng.choice(B, size=2, replace=False)]
+    layers_for = {b: (list(range(L)) if b in full else [int(rng.integers(0, L))]) for b in range(B)}
+    worst = decode_sampled(pool, seed, lens, tables, q, out, layers_for, bt)
+    assert worst <= TOL, worst
+    pool.close()
+    del pool
+    torch.cuda.empty_cache()
+
+
+def test_resume_burst_full_size(P, cuda_dev):
+    n, T, bt, seed = 8, 32768, 16, 3
+    nb = 2 * n * (T // bt)
+    pool = P.Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=n * T * 96 * 1024 + 4096,
+                  max_sessions=2 * n, max_batch=8, max_context=T, alloc_seed=seed)
+    sids = [pool.session_create_paused(T, T) for _ in range(n)]
+    for s in sids:
+        synth.fill_image_torch(pool.image(s), seed, s, L, HKV, D, T)
+    st = torch.cuda.Stream()
+    for s in sids:
+        pool.session_resume(s, st)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    ref = oracle.FreeList(nb, seed)
+    hv = pool.hot_view()
+    for s in sids:
+        row = pool.session_block_table(s)
+        assert row == list(ref.pop(T // bt))                 # placement bit-exact
+        blocks = hv[torch.as_tensor(row, device=cuda_dev, dtype=torch.int64)]
+        as_img = blocks.permute(1, 2, 3, 0, 4, 5).reshape(L, 2, HKV, T, D)
+        assert torch.equal(as_img.view(torch.int16), pool.image(s).view(torch.int16))
+    # host re-check of a sampled range through the oracle's unpack
+    s = sids[5]
+    Ts = 1000
+    img_h = bits(pool.image(s)[:, :, :, :Ts])
+    row = pool.session_block_table(s)[: -(-Ts // bt)]
+    small = np.zeros((len(row), L, 2, HKV, bt, D), dtype=np.uint16)
+    oracle.unpack(img_h, Ts, np.arange(len(row), dtype=np.int32), small)
+    got = bits(hv[torch.as_tensor(row, device=cuda_dev, dtype=torch.int64)])
+    for j in range(len(row)):
+        m = min(bt, Ts - j * bt)
+        assert np.array_equal(got[j, :, :, :, :m], small[j, :, :, :, :m])
+    # reverse: fresh sessions filled by append, packed into their images
+    for s in sids:
+        pool.session_destroy(s)
+    k, v = synth.kv_logical_torch(seed, 0, range(L), HKV, D, 0, T, cuda_dev)
+    kk, vv = k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+    fresh = [pool.session_create(T) for _ in range(n)]
+    for s in fresh:
+        pool.session_append(s, kk, vv, st)
+        pool.session_pause(s, st)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    for s in fresh:
+        img = pool.image(s)
+        assert torch.equal(img[:, 0].view(torch.int16), k.view(torch.int16))
+        assert torch.equal(img[:, 1].view(torch.int16), v.view(torch.int16))
+    assert pool.stats()["bytes_packed"] == n * T * 96 * 1024
+    pool.close()
+    del pool, k, v, kk, vv
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("B,T,bt,all_layers", [(1, 131072, 16, False), (1, 1024, 16, True),
+                                               (256, 1024, 16, False), (8, 16384, 64, False),
+                                               (32, 4096, 64, True)])
+def test_sweep_points(P, cuda_dev, B, T, bt, all_layers):
+    seed = 11 + B + bt
+    lens = np.full(B, T, dtype=np.int64)
+    lens[0] = T - 5                                     # one ragged tail
+    nb = int(sum(-(-int(t) // bt) for t in lens)) + 8
+    pool = P.Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,
+                  max_sessions=4, max_batch=L * B, max_context=T)
+    tables = synth.random_block_tables(seed, lens, bt, nb)
+    synth.fill_hot_pool_torch(pool.hot, seed, list(range(B)), lens, tables, L, HKV, D, bt,
+                              chunk_blocks=32)
+    q = synth.queries_torch(seed, range(B), range(L), HQ, D, cuda_dev).contiguous()
+    tab_d = torch.as_tensor(tables, device=cuda_dev)
+    len_d = torch.as_tensor(lens.astype(np.int32), device=cuda_dev)
+    out = torch.full((L, B, HQ, D), float("nan"), dtype=torch.float32, device=cuda_dev)
+    if all_layers:
+        pool.decode_attention(-1, q, tab_d, len_d, B, tab_d.shape[1], 1 / math.sqrt(D), out)
+    else:
+        for l in range(L):
+            pool.decode_attention(l, q[l], tab_d, len_d, B, tab_d.shape[1], 1 / math.sqrt(D),
+                                  out[l])
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    assert torch.isfinite(out).all()
+    rng = np.random.default_rng(seed)
+    picks = sorted(set([0, B - 1] + [int(x) for x in rng.integers(0, B, size=2)]))
+    layers_for = {b: sorted(set(int(x) for x in rng.integers(0, L, size=2))) for b in picks}
+    worst = decode_sampled(pool, seed, lens, tables, q, out, layers_for, bt)
+    assert worst <= TOL, worst
+    pool.close()
+    del pool
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("T", [1024, 131072])
+def test_resume_sweep_points(P, cuda_dev, T):
+    bt, seed = 16, 21
+    nb = T // bt + 64
+    pool = P.Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=T * 96 * 1024 + 4096,
+                  max_sessions=2, max_batch=4, max_context=T, alloc_seed=seed)
+    s = pool.session_create_paused(T, T)
+    synth.fill_image_torch(pool.image(s), seed, s, L, HKV, D, T)
+    pool.session_resume(s)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    row = pool.session_block_table(s)
+    assert row == list(oracle.FreeList(nb, seed).pop(T // bt))
+    blocks = pool.hot_view()[torch.as_tensor(row, device=cuda_dev, dtype=torch.int64)]
+    as_img = blocks.permute(1, 2, 3, 0, 4, 5).reshape(L, 2, HKV, T, D)
+    assert torch.equal(as_img.view(torch.int16), pool.image(s).view(torch.int16))
+    pool.close()
+    del pool, blocks, as_img
+    torch.cuda.empty_cache()

@@ -1,0 +1,91 @@
+"""The agentic trace driver end to end on a small configuration.
+
+Sessions cycle through resume -> turn append -> decode burst -> pause many
+times on two streams. At sampled steps the decode outputs are checked against
+the oracle (values regenerated on the host from their logical positions),
+and at the end every cold image must hold exactly the session's logical KV
+for the tokens it has packed.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+
+
+def test_small_trace_parity(cuda_dev):
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool, kvtier
+    from paper_2609_25782_gb300 import trace as tr
+
+    cfg = tr.TraceConfig(sessions=6, t0_min=100, t0_max=700, burst_mean=8.0, pause_mean_s=0.6,
+                         append_median=40.0, append_sigma=1.0, append_max=300, active_cap=2,
+                         steps=150, dt_s=0.1, layers=2, seed=5)
+    trace = tr.generate(cfg)
+    plan = tr.plan(cfg, trace)
+    assert plan["counts"]["pauses"] >= 10
+    L, Hkv, Hq, D, bt = cfg.layers, cfg.num_kv_heads, cfg.num_q_heads, 128, cfg.block_tokens
+    nb = plan["peak_blocks"] + 40
+    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=plan["cold_bytes"] + 4096,
+                max_sessions=cfg.sessions, max_batch=cfg.active_cap,
+                max_context=plan["max_context"], alloc_seed=9)
+    for i, t in enumerate(trace):
+        sid = pool.session_create_paused(plan["caps"][i], t.t0)
+        assert sid == i
+        synth.fill_image_torch(pool.image(sid), cfg.seed, sid, L, Hkv, D, t.t0)
+
+    def kv_source(sid, t0, t1):
+        k, v = synth.kv_logical_torch(cfg.seed, sid, range(L), Hkv, D, t0, t1, cuda_dev)
+        return k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+
+    q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(L), Hq, D, cuda_dev)
+    out = torch.empty(L, cfg.active_cap, Hq, D, dtype=torch.float32, device=cuda_dev)
+    max_blocks = -(-plan["max_context"] // bt)
+    tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=cuda_dev)
+    seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=cuda_dev)
+    dstream, mstream = torch.cuda.Stream(), torch.cuda.Stream()
+    checked = []
+
+    def on_step(k, members):
+        if k % 13 != 5:
+            return
+        torch.cuda.synchronize()
+        got = out[:, :len(members)].double().cpu().numpy()
+        lens = [int(kvtier.session_info(pool.handle, m).tokens) for m in members]
+        tab = np.full((len(members), max_blocks), -1, dtype=np.int32)
+        for r, m in enumerate(members):
+            row = pool.session_block_table(m)
+            tab[r, :len(row)] = row
+        hot = synth.hot_pool_np(cfg.seed, members, lens, tab, nb, L, Hkv, D, bt)
+        qh = q[:, :len(members)].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+        ref = oracle.paged_decode(hot, qh, tab, lens, 1 / math.sqrt(D), Hq)
+        err = np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref)))
+        assert err <= TOL, f"step {k}: scaled error {err}"
+        checked.append(k)
+
+    d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
+                       decode_stream=dstream, mig_stream=mstream, tables=tables,
+                       seq_lens=seq_lens, max_blocks=max_blocks, on_step=on_step)
+    d.run()
+    torch.cuda.synchronize()
+    assert len(checked) >= 5
+    assert d.counts == plan["counts"]          # same schedule as the dry run
+    assert pool.check_device() == 0
+    st = pool.stats()
+    assert st["pauses"] == plan["counts"]["pauses"] and st["resumes"] == plan["counts"]["resumes"]
+    # every image holds the session's logical KV for its packed prefix
+    for i in range(cfg.sessions):
+        info = kvtier.session_info(pool.handle, i)
+        n = int(info.cold_valid)
+        img = pool.image(i)[:, :, :, :n].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+        k, v = synth.session_kv_np(cfg.seed, i, range(L), Hkv, D, n)
+        assert np.array_equal(img[:, 0], k) and np.array_equal(img[:, 1], v)
+    pool.close()
