@@ -19,6 +19,7 @@ Under torchrun each rank runs an independent replica on its own sessions
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -45,6 +46,20 @@ def hbm_peak():
             return float(json.load(f)["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM, "fallback"
+
+
+def recorded_traffic():
+    """DRAM bytes per launch of the decode split kernel from the committed ncu
+    capture, or None when the kernel source changed since it was taken."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "decode_split_kernel.traffic.json")) as f:
+            rec = json.load(f)
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+        return int(rec["dram_bytes_per_launch"])
+    except Exception:
+        return None
 
 
 def dist_env():
@@ -685,9 +700,12 @@ def main():
             "e2e": {"value": round(e2e, 1), "unit": "GB/s", "h2d_bytes_per_step": res["h2d"],
                     "d2h_bytes_per_step": res["d2h"]},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-                         "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4),
+                         "traffic": recorded_traffic() if headline else None,
                          "peak_kind": peak_kind,
-                         "kernel": "decode_split_kernel + decode_combine_kernel (one layer call)"},
+                         "kernel": "decode_split_kernel; events bracket each decode_attention "
+                                   "call (split kernel + its dependent combine)",
+                         "alg_bytes_per_launch": int(res["launch_alg_bytes"])},
             "cpu_baseline": cpu,
             "gpu_launches": 2 * nl * args.steps,
             "clocks": res["clocks"],
