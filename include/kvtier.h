@@ -170,6 +170,20 @@ int decode_attention(kv_pool *pool, int32_t layer, const void *q,
                      const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                      int32_t max_blocks, float scale, float *out, kv_stream_t stream);
 
+/* decode_attention with options. KV_DECODE_OVERLAP_PREVIOUS lets this
+ * call's split kernel start while the kernel just before it on the stream is
+ * still running (programmatic dependent launch): it reads block ids and
+ * prefetches K/V tiles at once, and waits for that kernel to finish before
+ * it reads q or writes out or the workspace. The caller promises that the
+ * kernel just before it on the stream (typically the previous layer's
+ * decode_attention call) does not write the hot arena, block_tables or
+ * seq_lens. flags = 0 is decode_attention. */
+#define KV_DECODE_OVERLAP_PREVIOUS 1u
+int decode_attention_ex(kv_pool *pool, int32_t layer, const void *q,
+                        const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
+                        int32_t max_blocks, float scale, float *out, uint32_t flags,
+                        kv_stream_t stream);
+
 /* Data path 4 with write-on-evict (Section 3, "Memory hierarchy and write
  * policy"): copy tokens [cold_valid, T) of an ACTIVE session into its
  * image, set cold_valid = T, return its hot blocks to the end of the free

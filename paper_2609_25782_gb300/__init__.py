@@ -102,9 +102,14 @@ class Pool:
                                     stream)
 
     def decode_attention(self, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
-                         scale: float, out, stream=None) -> None:
-        kvtier.decode_attention(self.handle, layer, q, block_tables, seq_lens, B, max_blocks,
-                                scale, out, stream)
+                         scale: float, out, stream=None, overlap_previous: bool = False) -> None:
+        if overlap_previous:
+            kvtier.decode_attention_ex(self.handle, layer, q, block_tables, seq_lens, B,
+                                       max_blocks, scale, out, kvtier.KV_DECODE_OVERLAP_PREVIOUS,
+                                       stream)
+        else:
+            kvtier.decode_attention(self.handle, layer, q, block_tables, seq_lens, B, max_blocks,
+                                    scale, out, stream)
 
     def shuffle_free(self, seed: int) -> None:
         kvtier.kv_pool_shuffle_free(self.handle, seed)

@@ -210,6 +210,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 2)
     if (lane == 0)
         for (int k = 0; k < kStages && k < my_tiles; ++k) issue(k);
 
+    // Everything above reads only the hot pool, the block table and seq_lens.
+    // When this grid is launched as a programmatic dependent (the caller's
+    // overlap option) it may run while the previous decode call drains; Q is
+    // read, and partials/outputs written, only after that call completes.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+
     // Q^T fragments (mma B operand): head n = lane/4 of the group, dims
     // 16*ks + 2*(lane%4) + {0,1} and +8.
     uint32_t qb[8][2];
@@ -409,6 +415,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 2)
 // completion with griddepcontrol.wait, so its CTAs can already be resident
 // while K1 drains.
 __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a) {
+    asm volatile("griddepcontrol.launch_dependents;");   // a following overlapped call
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const int64_t row = blockIdx.x;                // lb * Hq + h
     const int lb = static_cast<int>(row / a.s.Hq);
@@ -605,25 +612,33 @@ cudaError_t prepare_kernels() {
                                 kDecodeSmem);
 }
 
-cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st) {
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st,
+                          bool overlap_previous) {
     // Every session of the batch has T <= max_blocks * bt, so its splits fit.
     const int splits = max_splits_for(static_cast<int64_t>(a.max_blocks) * a.s.bt);
     if (splits > a.max_splits) return cudaErrorInvalidValue;
-    dim3 grid(splits, a.s.Hkv, a.nlayers * a.B);
-    decode_split_kernel<<<grid, kDecodeWarps * 32, kDecodeSmem, st>>>(map, a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
-    cfg.blockDim = dim3(kDecodeWarps * 32);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_combine_kernel, a);
+
+    cudaLaunchConfig_t c1 = {};
+    c1.gridDim = dim3(splits, a.s.Hkv, a.nlayers * a.B);
+    c1.blockDim = dim3(kDecodeWarps * 32);
+    c1.dynamicSmemBytes = kDecodeSmem;
+    c1.stream = st;
+    c1.attrs = overlap_previous ? attr : nullptr;
+    c1.numAttrs = overlap_previous ? 1 : 0;
+    cudaError_t e = cudaLaunchKernelEx(&c1, decode_split_kernel, map, a);
+    if (e != cudaSuccess) return e;
+
+    cudaLaunchConfig_t c2 = {};
+    c2.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
+    c2.blockDim = dim3(kDecodeWarps * 32);
+    c2.dynamicSmemBytes = 0;
+    c2.stream = st;
+    c2.attrs = attr;
+    c2.numAttrs = 1;
+    return cudaLaunchKernelEx(&c2, decode_combine_kernel, a);
 }
 
 static unsigned mig_grid(int64_t items, int num_sms) {

@@ -99,7 +99,10 @@ struct GatherArgs {
 // Host launchers (kernels.cu). Each returns the launch's CUDA status.
 bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why);
 cudaError_t prepare_kernels();  // per-device function attributes
-cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st);
+// overlap_previous: launch the split kernel as a programmatic dependent of the
+// previous kernel on the stream (see decode_attention_ex).
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st,
+                          bool overlap_previous);
 cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);

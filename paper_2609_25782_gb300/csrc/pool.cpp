@@ -443,6 +443,15 @@ int session_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_
 int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
                      const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
                      float *out, kv_stream_t stream_) {
+    return decode_attention_ex(p, layer, q, block_tables, seq_lens, B, max_blocks, scale, out, 0u,
+                               stream_);
+}
+
+int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
+                        const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
+                        float *out, uint32_t flags, kv_stream_t stream_) {
+    if (flags & ~static_cast<uint32_t>(KV_DECODE_OVERLAP_PREVIOUS))
+        return fail(KV_ERR_INVALID_ARG, "unknown decode flag");
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
     if (!q || !block_tables || !seq_lens || !out) return fail(KV_ERR_INVALID_ARG, "null pointer");
@@ -476,7 +485,8 @@ int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *bl
     a.scale_log2 = scale * 1.4426950408889634f;
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
-    int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, st); });
+    const bool overlap = (flags & KV_DECODE_OVERLAP_PREVIOUS) != 0;
+    int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, st, overlap); });
     if (rc) return rc;
     p->stats.decodes += 1;
     return KV_OK;

@@ -36,7 +36,10 @@ EXPORTS = [
     "session_info", "session_block_table", "kv_pool_batch_tables", "kv_pool_shuffle_free",
     "kv_pool_free_list", "kv_pool_get_stats", "kv_pool_check_device",
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
+    "decode_attention_ex",
 ]
+
+KV_DECODE_OVERLAP_PREVIOUS = 1
 
 KV_NOALLOC_SCRATCH_BYTES = 48 << 20
 
@@ -87,6 +90,7 @@ def _load():
         "session_destroy": [p, i32],
         "session_append": [p, i32, p, p, i32, p],
         "decode_attention": [p, i32, p, p, p, i32, i32, C.c_float, p, p],
+        "decode_attention_ex": [p, i32, p, p, p, i32, i32, C.c_float, p, C.c_uint32, p],
         "session_pause": [p, i32, p],
         "session_resume": [p, i32, p],
         "session_ready_event": [p, i32, C.POINTER(p)],
@@ -188,6 +192,13 @@ def decode_attention(pool: int, layer: int, q, block_tables, seq_lens, B: int, m
     _check(lib.decode_attention(pool, layer, _addr(q), _addr(block_tables), _addr(seq_lens), B,
                                 max_blocks, scale, _addr(out), _stream(stream)),
            "decode_attention")
+
+
+def decode_attention_ex(pool: int, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
+                        scale: float, out, flags: int, stream=None) -> None:
+    _check(lib.decode_attention_ex(pool, layer, _addr(q), _addr(block_tables), _addr(seq_lens), B,
+                                   max_blocks, scale, _addr(out), flags, _stream(stream)),
+           "decode_attention_ex")
 
 
 def session_pause(pool: int, sid: int, stream=None) -> None:

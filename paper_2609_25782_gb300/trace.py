@@ -199,9 +199,11 @@ class TraceDriver:
                 kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
                                             self.seq_lens, self.dstream)
                 for l in range(cfg.layers):
-                    kvtier.decode_attention(self.pool, l, self.q[l], self.tables, self.seq_lens,
-                                            B, self.max_blocks, 1 / math.sqrt(128), self.out[l],
-                                            self.dstream)
+                    # layer l > 0 follows layer l-1's call, which writes only `out`
+                    kvtier.decode_attention_ex(
+                        self.pool, l, self.q[l], self.tables, self.seq_lens, B, self.max_blocks,
+                        1 / math.sqrt(128), self.out[l],
+                        kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 else 0, self.dstream)
                 end.record(self.dstream)
                 self.last_decode_ev = end
                 self.step_events.append((start, end, B))

@@ -139,6 +139,35 @@ def test_decode_independent_of_batch_and_placement(pkg):
     assert np.array_equal(moved, full)
 
 
+def test_overlapped_calls_bit_identical(pkg):
+    """Per-layer calls launched with KV_DECODE_OVERLAP_PREVIOUS (each one
+    overlapping the previous call's end) give the same bits as serialised
+    calls, over several rounds on one stream."""
+    lens = [77, 1500, 4100, 9000, 33]
+    L = 6
+    pool, sess, tables, q = direct_case(pkg, lens, L=L, seed=12)
+    dev = torch.device("cuda:0")
+    t = torch.as_tensor(tables, device=dev)
+    s = torch.as_tensor(np.asarray(lens, dtype=np.int32), device=dev)
+    st = torch.cuda.Stream()
+    outs = []
+    for overlap in (False, True, True):
+        out = torch.full((L, len(lens), 32, 128), float("nan"), dtype=torch.float32, device=dev)
+        for rnd in range(2):
+            for l in range(L):
+                pool.decode_attention(l, q[l].contiguous(), t, s, len(lens), t.shape[1],
+                                      1 / math.sqrt(128), out[l], st,
+                                      overlap_previous=overlap and (l > 0 or rnd > 0))
+        torch.cuda.synchronize()
+        outs.append(out.clone())
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+    ref = oracle.paged_decode(host_hot(pool, 12, sess, lens, tables),
+                              q.cpu().view(torch.int16).numpy().view(np.uint16), tables, lens,
+                              1 / math.sqrt(128), 32)
+    assert scaled_err(outs[1].double().cpu().numpy(), ref) <= TOL
+    assert pool.check_device() == 0
+
+
 def test_nan_tail_slots_do_not_leak(pkg):
     lens = [17, 100, 529]
     pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=6)
