@@ -62,6 +62,23 @@ def recorded_traffic():
         return None
 
 
+def replica_seed(seed: int, rank: int) -> int:
+    """Each rank serves its own sessions: disjoint seeded draws per rank."""
+    return seed + 1000 * rank
+
+
+def reduce_over_ranks(total_ms: float, e2e_ms: float, kv_bytes: float, device="cpu"):
+    """Max of the timed regions and sum of the bytes over all ranks (the
+    whole-job value divides the summed bytes by the slowest rank's time)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([total_ms, e2e_ms, kv_bytes], dtype=torch.float64, device=device)
+    mx, sm = t.clone(), t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(mx[1]), float(sm[2])
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -130,7 +147,7 @@ def decode_workload(args, rank: int):
     import synth
     from paper_2609_25782_gb300 import Pool
     dev = torch.device("cuda", torch.cuda.current_device())
-    s = args.seed + 1000 * rank
+    s = replica_seed(args.seed, rank)
     nl, B = args.layers, args.batch
     lens = synth.session_lengths(s, B, args.tmin, args.tmax, BT)
     nb = int(sum(-(-int(t) // BT) for t in lens)) + 64
@@ -349,7 +366,7 @@ def run_trace(args, rank):
     from paper_2609_25782_gb300 import Pool, kvtier
     from paper_2609_25782_gb300 import trace as tr
     dev = torch.device("cuda", torch.cuda.current_device())
-    cfg = tr.TraceConfig(seed=args.seed + 1000 * rank, steps=args.trace_steps)
+    cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -650,12 +667,8 @@ def main():
     total_ms = res["total_ms"]
     e2e_ms = res["e2e_ms"]
     if ws > 1:
-        t = torch.tensor([total_ms, e2e_ms, float(res["kv_bytes"])], device="cuda")
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = t.clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        total_ms, e2e_ms, all_kv = float(mx[0]), float(mx[1]), float(sm[2])
+        total_ms, e2e_ms, all_kv = reduce_over_ranks(total_ms, e2e_ms, float(res["kv_bytes"]),
+                                                     device="cuda")
     else:
         all_kv = float(res["kv_bytes"])
     value = all_kv * args.steps / (total_ms * 1e-3) / 1e9
@@ -671,7 +684,7 @@ def main():
         res["pool"] = keep
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(res, args.seed + 1000 * rank)
+        cpu = cpu_baseline(res, replica_seed(args.seed, rank))
     res["pool"].close()
     del res["pool"]
     torch.cuda.empty_cache()
