@@ -358,9 +358,12 @@ def run_migration(args, rank):
     }
 
 
-def run_trace(args, rank):
+def run_trace(args, rank, lru_factor: float = 0.0):
     """Agentic trace: 48 sessions, N_a = 16, decode on one stream and
-    pack/unpack on another; step p50/p99 from events on the decode stream."""
+    pack/unpack on another; step p50/p99 from events on the decode stream.
+    lru_factor > 0: block residency mode with a hot pool of lru_factor times
+    the simple mode's peak; its statistics must equal the host dry run's."""
+    import dataclasses
     import torch
     import synth
     from paper_2609_25782_gb300 import Pool, kvtier
@@ -370,9 +373,15 @@ def run_trace(args, rank):
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
+    dry = None
+    if lru_factor > 0:
+        cfg = dataclasses.replace(cfg, lru=True)
+        nb = int(plan["peak_blocks"] * lru_factor)
+        dry = tr.plan(cfg, trace, hot_blocks=nb)["stats"]
     pool = Pool(num_layers=cfg.layers, num_hot_blocks=nb, cold_bytes=plan["cold_bytes"] + 4096,
                 max_sessions=cfg.sessions, max_batch=cfg.active_cap,
-                max_context=plan["max_context"], alloc_seed=cfg.seed, device=dev.index)
+                max_context=plan["max_context"], alloc_seed=cfg.seed, device=dev.index,
+                lru_residency=cfg.lru)
     for i, t in enumerate(trace):
         sid = pool.session_create_paused(plan["caps"][i], t.t0)
         synth.fill_image_torch(pool.image(sid), cfg.seed, sid, cfg.layers, cfg.num_kv_heads, D,
@@ -419,7 +428,20 @@ def run_trace(args, rank):
     def pct(p):
         return steps_ms[min(len(steps_ms) - 1, int(round(p / 100 * (len(steps_ms) - 1))))]
 
+    extra = {}
+    if cfg.lru:
+        hit, miss = st["resume_blocks_hit"], st["resume_blocks_missed"]
+        extra = {"mode": "LRU block residency, write-on-evict", "hot_blocks": nb,
+                 "hot_vs_simple_peak": lru_factor,
+                 "resume_hit_rate": round(hit / max(1, hit + miss), 4),
+                 "blocks_evicted": st["blocks_evicted"],
+                 "cold_write_gb": round(st["bytes_packed"] / 1e9, 2),
+                 "cold_read_gb": round(st["bytes_unpacked"] / 1e9, 2),
+                 "matches_dry_run": all(st[k] == dry[k] for k in (
+                     "bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
+                     "resume_blocks_missed", "resumes", "pauses"))}
     return {
+        **extra,
         "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
         "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
         "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2),
@@ -690,6 +712,7 @@ def main():
     torch.cuda.empty_cache()
     if secondary is not None and not args.no_trace:
         secondary["trace"] = run_trace(args, rank)
+        secondary["trace_lru"] = run_trace(args, rank, lru_factor=1.5)
     nl, nbatch = args.layers, args.batch
     headline = (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2)
     shape = ("Qwen3-Coder-30B-A3B KV shape (48 layers, Hq 32, Hkv 4, D 128, 16-token blocks), "

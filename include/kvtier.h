@@ -68,6 +68,28 @@ enum { KV_SESSION_FREE = 0, KV_SESSION_ACTIVE = 1, KV_SESSION_PAUSED = 2 };
  * the host logic (placement, states, errors) on machines without a GPU. */
 #define KV_POOL_HOST_LOGIC_ONLY 1u
 
+/* Pool flag: block residency with LRU eviction (Section 3, "Eviction, resume
+ * and decode"; Section 4: each 1.5 MiB block is resident in HBM, the cold
+ * tier, or both, with write-back LRU). In this mode
+ *  - session_pause moves nothing: a paused session's blocks stay hot and age;
+ *  - when an allocation finds no free block, the least recently used hot
+ *    blocks are evicted (sessions ordered by last use, i.e. the last append,
+ *    resume or kv_pool_batch_tables that named them; ties by session id;
+ *    within a session, ascending block index). Active blocks are not pinned;
+ *    the sessions the current call works on are never its victims;
+ *  - an evicted block is written to the session's image only for the tokens
+ *    the image does not hold yet, so every token is written at most once
+ *    (write-on-evict, Section 3, "Memory hierarchy and write policy");
+ *  - session_resume fetches only the blocks that are no longer hot (the
+ *    others count as resume hits), and kv_pool_batch_tables first fetches
+ *    any evicted block of its sessions;
+ *  - evicted slots go to the end of the free list, in eviction order, and the
+ *    call's allocations pop from the end.
+ * Any call that allocates may evict blocks of any other session, so order it
+ * after the decode work that still reads the pool (evictions wait for the
+ * victims' own appends and resumes by themselves). */
+#define KV_POOL_LRU_RESIDENCY 2u
+
 typedef struct kv_pool_config {
     int32_t num_layers;     /* L  (48 for Qwen3-Coder-30B-A3B)             */
     int32_t num_q_heads;    /* Hq (32); Hq / Hkv must be 1, 2, 4 or 8      */
@@ -83,13 +105,13 @@ typedef struct kv_pool_config {
     int64_t cold_bytes;     /* bytes in the cold arena                      */
     void *cold_base;        /* device, 256-B aligned                        */
     uint64_t alloc_seed;    /* seeds the shuffle of the initial free list   */
-    uint32_t flags;         /* 0 or KV_POOL_HOST_LOGIC_ONLY                 */
+    uint32_t flags;         /* KV_POOL_HOST_LOGIC_ONLY | KV_POOL_LRU_RESIDENCY */
     uint32_t reserved;
 } kv_pool_config;
 
 typedef struct kv_session_info {
     int32_t state;       /* KV_SESSION_*                                   */
-    int32_t num_blocks;  /* hot blocks held (0 when paused)                */
+    int32_t num_blocks;  /* hot blocks held (simple mode: 0 when paused)   */
     int64_t tokens;      /* T: tokens in the session's KV                  */
     int64_t capacity;    /* T_cap of its cold image                        */
     int64_t cold_valid;  /* tokens already valid in the cold image         */
@@ -104,6 +126,9 @@ typedef struct kv_pool_stats {
     int64_t bytes_packed;     /* image bytes copied hot -> cold (path 4)   */
     int64_t bytes_appended;   /* KV bytes written by session_append        */
     int64_t resumes, pauses, appends, decodes;
+    int64_t blocks_evicted;       /* residency mode: blocks evicted            */
+    int64_t resume_blocks_hit;    /* residency mode: still hot at resume       */
+    int64_t resume_blocks_missed; /* residency mode: fetched at resume         */
 } kv_pool_stats;
 
 /* Create a pool over caller-owned arenas. The hot free list starts as

@@ -22,7 +22,8 @@ class Pool:
     def __init__(self, *, num_layers: int, num_hot_blocks: int, cold_bytes: int,
                  num_q_heads: int = 32, num_kv_heads: int = 4, head_dim: int = 128,
                  block_tokens: int = 16, max_sessions: int = 64, max_batch: int = 64,
-                 max_context: int = 32768, alloc_seed: int = 0, device: int = 0):
+                 max_context: int = 32768, alloc_seed: int = 0, device: int = 0,
+                 lru_residency: bool = False):
         import torch
         self.device = torch.device("cuda", device)
         self.L, self.Hq, self.Hkv, self.D, self.bt = (num_layers, num_q_heads, num_kv_heads,
@@ -41,7 +42,8 @@ class Pool:
                                  block_tokens=block_tokens, max_sessions=max_sessions,
                                  max_batch=max_batch, device=device, max_context=max_context,
                                  num_hot_blocks=num_hot_blocks, hot_base=self.hot,
-                                 cold_bytes=cold_bytes, cold_base=self.cold, alloc_seed=alloc_seed)
+                                 cold_bytes=cold_bytes, cold_base=self.cold, alloc_seed=alloc_seed,
+                                 flags=kvtier.KV_POOL_LRU_RESIDENCY if lru_residency else 0)
         self.handle = kvtier.kv_pool_create(cfg)
         self.max_context = max_context
 

@@ -532,6 +532,45 @@ __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
     }
 }
 
+// K3'/K4': block-granular moves for the residency mode: one warp per
+// (job, layer, K|V, kv-head) run; a job moves tokens [t0, t1) of one block.
+template <bool kPack>
+__global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__ BlockJobs a) {
+    const Shape sh = a.s;
+    const int runs = sh.L * 2 * sh.Hkv;
+    const int items = a.n * runs;
+    const int lane = threadIdx.x & 31;
+    const int nwarps = (gridDim.x * blockDim.x) >> 5;
+    for (int it = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; it < items; it += nwarps) {
+        const int jb = it / runs;
+        const int c = it - jb * runs;
+        const BlockJob &b = a.job[jb];
+        if (b.slot < 0 || b.slot >= sh.num_blocks || b.t0 < 0 || b.t1 > sh.bt) {
+            if (lane == 0) atomicOr(a.err, kErrBadBlock);
+            continue;
+        }
+        uint8_t *hp = a.hot + ((static_cast<int64_t>(b.slot) * runs + c) * sh.bt + b.t0) * kRowBytes;
+        uint8_t *ip = b.img + (static_cast<int64_t>(c) * b.T_cap + static_cast<int64_t>(b.j) * sh.bt +
+                               b.t0) * kRowBytes;
+        const uint4 *src = reinterpret_cast<const uint4 *>(kPack ? hp : ip);
+        uint4 *dst = reinterpret_cast<uint4 *>(kPack ? ip : hp);
+        const int units = (b.t1 - b.t0) * (kRowBytes / 16);
+        for (int u0 = 0; u0 < units; u0 += 32 * 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < units) v[k] = ld_stream(src + u);
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < units) dst[u] = v[k];
+            }
+        }
+    }
+}
+
 // K5: one warp per (layer, token): the token's K and V rows for all kv-heads
 // are 2 x Hkv*256 contiguous bytes in the source; each 256-byte head row goes
 // to its (layer, K|V, head) run of the tail block.
@@ -667,6 +706,16 @@ cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st) {
     int64_t blocks = (warps + 7) / 8;
     if (blocks > static_cast<int64_t>(num_sms) * 8) blocks = static_cast<int64_t>(num_sms) * 8;
     append_kernel<<<static_cast<unsigned>(blocks < 1 ? 1 : blocks), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, cudaStream_t st) {
+    if (a.n <= 0) return cudaSuccess;
+    const unsigned grid = mig_grid(static_cast<int64_t>(a.n) * a.s.L * 2 * a.s.Hkv, num_sms);
+    if (pack)
+        block_jobs_kernel<true><<<grid, 256, 0, st>>>(a);
+    else
+        block_jobs_kernel<false><<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

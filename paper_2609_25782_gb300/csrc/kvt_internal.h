@@ -75,6 +75,23 @@ struct AppendArgs {
     Shape s;
 };
 
+// One block move between a hot slot and a session image: tokens [t0, t1) of
+// logical block j (all layers, K and V, all kv-heads).
+struct BlockJob {
+    uint8_t *img;             // the session's image base
+    int64_t T_cap;
+    int32_t slot, j, t0, t1;
+};
+constexpr int kBlockJobsMax = 960;   // keeps the parameter block under 32 KB
+struct BlockJobs {
+    uint8_t *hot;
+    int32_t *err;
+    Shape s;
+    int32_t n;
+    int32_t pad;
+    BlockJob job[kBlockJobsMax];
+};
+
 constexpr int kTableWriteMax = 2048;
 struct TableWriteArgs {
     int32_t *dst;
@@ -106,6 +123,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStrea
 cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, cudaStream_t st);
 cudaError_t launch_table_write(const TableWriteArgs &a, cudaStream_t st);
 cudaError_t launch_gather(const GatherArgs &a, cudaStream_t st);
 

@@ -10,6 +10,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <set>
 #include <string>
 #include <vector>
 
@@ -47,11 +48,20 @@ struct Session {
     int32_t state = KV_SESSION_FREE;
     int64_t T = 0, cap = 0, cold_valid = 0;
     int64_t img_off = -1, img_bytes = 0;
-    std::vector<int32_t> blocks;
+    std::vector<int32_t> blocks;      // per logical block: hot slot, or -1 (residency mode)
+    std::vector<int16_t> img_tok;     // residency mode: tokens of block j held by the image
+    int64_t hot_count = 0;            // residency mode: blocks with a hot slot
+    uint64_t last_use = 0;            // residency mode: recency stamp
     cudaEvent_t ready = nullptr;
     bool ready_recorded = false;
     cudaEvent_t appended = nullptr;
     bool appended_recorded = false;
+};
+
+// A planned eviction: block j of session sid leaves hot slot `slot`; tokens
+// [t0, t1) are written to the image first (t0 == t1: the image has them).
+struct Victim {
+    int32_t sid, j, slot, t0, t1;
 };
 
 constexpr int kFenceSlots = 64;
@@ -108,6 +118,12 @@ struct kv_pool {
 
     kv_pool_stats stats{};
     int32_t inject_countdown = 0;
+
+    // Residency mode (KV_POOL_LRU_RESIDENCY): sessions holding hot blocks,
+    // ordered by (last use, sid); the first one is the least recently used.
+    bool lru = false;
+    uint64_t clock = 0;
+    std::set<std::pair<uint64_t, int32_t>> lru_set;
 
     // Every CUDA call of the pool goes through here: the failure-injection
     // hook fires first, then (unless the pool is host-logic only) the call.
@@ -197,6 +213,115 @@ struct kv_pool {
         return KV_OK;
     }
 
+    // ---- residency mode -------------------------------------------------
+    int32_t tokens_in_block(const Session &s, int64_t j) const {
+        const int64_t n = s.T - j * cfg.block_tokens;
+        return static_cast<int32_t>(n < cfg.block_tokens ? n : cfg.block_tokens);
+    }
+
+    void lru_out(int32_t sid) {
+        Session &s = sessions[sid];
+        if (s.hot_count > 0) lru_set.erase({s.last_use, sid});
+    }
+    void lru_in(int32_t sid) {
+        Session &s = sessions[sid];
+        if (s.hot_count > 0) lru_set.insert({s.last_use, sid});
+    }
+
+    // Least recently used hot blocks, outside `protect`, until `need` blocks
+    // would be free. Sessions in recency order; within one, ascending j.
+    bool plan_evict(int64_t need, const std::vector<int32_t> &protect, std::vector<Victim> &out) {
+        int64_t have = static_cast<int64_t>(free_list.size());
+        for (const auto &e : lru_set) {
+            if (have >= need) break;
+            const int32_t sid = e.second;
+            if (std::find(protect.begin(), protect.end(), sid) != protect.end()) continue;
+            const Session &s = sessions[sid];
+            for (size_t j = 0; j < s.blocks.size() && have < need; ++j) {
+                if (s.blocks[j] < 0) continue;
+                out.push_back({sid, static_cast<int32_t>(j), s.blocks[j], s.img_tok[j],
+                               tokens_in_block(s, static_cast<int64_t>(j))});
+                ++have;
+            }
+        }
+        return have >= need;
+    }
+
+    // The `need` slots the call will pop once the victims are pushed back:
+    // the free list grows by the victims (in order), pops come off its end.
+    std::vector<int32_t> peek_alloc(int64_t need, const std::vector<Victim> &v) const {
+        std::vector<int32_t> all(free_list);
+        for (const Victim &x : v) all.push_back(x.slot);
+        std::vector<int32_t> out(need);
+        for (int64_t i = 0; i < need; ++i) out[i] = all[all.size() - 1 - i];
+        return out;
+    }
+
+    // Device side of the victims: wait for their last writes, then write the
+    // tokens each image lacks.
+    int evict_device(const std::vector<Victim> &v, cudaStream_t st) {
+        std::vector<int32_t> seen;
+        for (const Victim &x : v) {
+            if (std::find(seen.begin(), seen.end(), x.sid) != seen.end()) continue;
+            seen.push_back(x.sid);
+            Session &s = sessions[x.sid];
+            int rc = KV_OK;
+            if (s.appended_recorded)
+                rc = cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s.appended, 0); });
+            if (!rc && s.ready_recorded)
+                rc = cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s.ready, 0); });
+            if (rc) return rc;
+        }
+        std::vector<kvt::BlockJob> jobs;
+        for (const Victim &x : v)
+            if (x.t1 > x.t0) jobs.push_back(job_for(x.sid, x.j, x.slot, x.t0, x.t1));
+        return run_jobs(jobs, true, st);
+    }
+
+    void evict_commit(const std::vector<Victim> &v) {
+        for (const Victim &x : v) {
+            Session &s = sessions[x.sid];
+            lru_out(x.sid);
+            if (x.t1 > x.t0) stats.bytes_packed += static_cast<int64_t>(x.t1 - x.t0) * token_bytes;
+            s.img_tok[x.j] = static_cast<int16_t>(x.t1);
+            s.blocks[x.j] = -1;
+            s.hot_count -= 1;
+            lru_in(x.sid);
+            free_list.push_back(x.slot);
+            stats.blocks_evicted += 1;
+            stats.free_blocks += 1;
+            stats.used_blocks -= 1;
+        }
+    }
+
+    kvt::BlockJob job_for(int32_t sid, int32_t j, int32_t slot, int32_t t0, int32_t t1) const {
+        const Session &s = sessions[sid];
+        kvt::BlockJob b;
+        b.img = static_cast<uint8_t *>(cfg.cold_base) + s.img_off;
+        b.T_cap = s.cap;
+        b.slot = slot;
+        b.j = j;
+        b.t0 = t0;
+        b.t1 = t1;
+        return b;
+    }
+
+    int run_jobs(const std::vector<kvt::BlockJob> &jobs, bool pack, cudaStream_t st) {
+        for (size_t i = 0; i < jobs.size(); i += kvt::kBlockJobsMax) {
+            kvt::BlockJobs a;
+            a.hot = static_cast<uint8_t *>(cfg.hot_base);
+            a.err = d_err;
+            a.s = shape;
+            a.n = static_cast<int32_t>(std::min<size_t>(kvt::kBlockJobsMax, jobs.size() - i));
+            a.pad = 0;
+            std::copy(jobs.begin() + i, jobs.begin() + i + a.n, a.job);
+            int rc = cuda(pack ? "pack launch" : "unpack launch",
+                          [&] { return kvt::launch_block_jobs(a, pack, num_sms, st); });
+            if (rc) return rc;
+        }
+        return KV_OK;
+    }
+
     kvt::MigArgs mig_args(int32_t sid, const Session &s) const {
         kvt::MigArgs m;
         m.table = d_tables + static_cast<int64_t>(sid) * table_stride;
@@ -253,6 +378,7 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
     kv_pool *p = new kv_pool;
     p->cfg = c;
     p->host_only = host_only;
+    p->lru = (c.flags & KV_POOL_LRU_RESIDENCY) != 0;
     p->token_bytes = kv_token_bytes(&c);
     p->block_bytes = kv_block_bytes(&c);
     p->table_stride = static_cast<int32_t>((c.max_context + c.block_tokens - 1) / c.block_tokens);
@@ -351,6 +477,12 @@ static int create_session(kv_pool *p, int64_t max_tokens, int64_t tokens, int32_
     s.cold_valid = tokens;
     s.img_off = off;
     s.img_bytes = bytes;
+    if (p->lru && tokens > 0) {   // the image holds every block, none is hot
+        const int64_t nb = (tokens + p->cfg.block_tokens - 1) / p->cfg.block_tokens;
+        s.blocks.assign(nb, -1);
+        s.img_tok.resize(nb);
+        for (int64_t j = 0; j < nb; ++j) s.img_tok[j] = static_cast<int16_t>(p->tokens_in_block(s, j));
+    }
     p->stats.cold_bytes_used = p->cold_used;
     *sid_out = sid;
     return KV_OK;
@@ -369,9 +501,15 @@ int session_destroy(kv_pool *p, int32_t sid) {
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     Session *s = p->session(sid);
     if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
-    for (int32_t b : s->blocks) p->free_list.push_back(b);
-    p->stats.free_blocks += static_cast<int64_t>(s->blocks.size());
-    p->stats.used_blocks -= static_cast<int64_t>(s->blocks.size());
+    if (p->lru) p->lru_out(sid);
+    int64_t freed = 0;
+    for (int32_t b : s->blocks)
+        if (b >= 0) {
+            p->free_list.push_back(b);
+            ++freed;
+        }
+    p->stats.free_blocks += freed;
+    p->stats.used_blocks -= freed;
     p->cold_release(s->img_off, s->img_bytes);
     p->stats.cold_bytes_used = p->cold_used;
     cudaEvent_t ready = s->ready, appended = s->appended;
@@ -387,12 +525,193 @@ static int ensure_event(kv_pool *p, cudaEvent_t *ev) {
                    [&] { return cudaEventCreateWithFlags(ev, cudaEventDisableTiming); });
 }
 
+// ---- residency mode (KV_POOL_LRU_RESIDENCY) --------------------------------
+
+static int wait_event(kv_pool *p, cudaStream_t st, cudaEvent_t ev) {
+    return p->cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, ev, 0); });
+}
+
+// Append with residency: a tail block that was evicted comes back first,
+// new blocks come from the free list or from evicting LRU blocks.
+static int lru_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_t n,
+                      cudaStream_t st) {
+    Session *s = &p->sessions[sid];
+    if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "append to a paused session");
+    if (n < 1) return fail(KV_ERR_INVALID_ARG, "n must be >= 1");
+    if (!p->host_only && (!k || !v)) return fail(KV_ERR_INVALID_ARG, "null k or v");
+    if (s->T + n > s->cap) return fail(KV_ERR_INVALID_ARG, "append past the session capacity");
+    const int bt = p->cfg.block_tokens;
+    const int64_t have = static_cast<int64_t>(s->blocks.size());
+    const int64_t tail = s->T > 0 ? (s->T - 1) / bt : -1;
+    const bool refetch = (s->T % bt) != 0 && tail >= 0 && s->blocks[tail] < 0;
+    const int64_t fresh_n = (s->T + n + bt - 1) / bt - have;
+    const int64_t need = (refetch ? 1 : 0) + fresh_n;
+    std::vector<Victim> vic;
+    if (!p->plan_evict(need, {sid}, vic))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "no block can be evicted for the append");
+    const std::vector<int32_t> got = p->peek_alloc(need, vic);
+
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    int rc = ensure_event(p, &s->appended);
+    if (!rc && s->ready_recorded) rc = wait_event(p, st, s->ready);
+    if (!rc) rc = p->evict_device(vic, st);
+    if (!rc && refetch) {
+        rc = p->run_jobs({p->job_for(sid, static_cast<int32_t>(tail), got[0], 0,
+                                     p->tokens_in_block(*s, tail))}, false, st);
+        if (!rc) rc = p->write_table(sid, &got[0], tail, 1, st);
+    }
+    if (!rc && fresh_n > 0)
+        rc = p->write_table(sid, got.data() + (refetch ? 1 : 0), have, fresh_n, st);
+    if (!rc) {
+        kvt::AppendArgs a;
+        a.k = static_cast<const uint8_t *>(k);
+        a.v = static_cast<const uint8_t *>(v);
+        a.table = p->d_tables + static_cast<int64_t>(sid) * p->table_stride;
+        a.hot = static_cast<uint8_t *>(p->cfg.hot_base);
+        a.pos0 = s->T;
+        a.n = n;
+        a.err = p->d_err;
+        a.s = p->shape;
+        rc = p->cuda("append launch", [&] { return kvt::launch_append(a, p->num_sms, st); });
+    }
+    if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->appended, st); });
+    if (rc) return rc;   // host state untouched
+
+    p->evict_commit(vic);
+    p->free_list.resize(p->free_list.size() - need);
+    p->lru_out(sid);
+    if (refetch) {
+        s->blocks[tail] = got[0];
+        s->hot_count += 1;
+        p->stats.bytes_unpacked += p->tokens_in_block(*s, tail) * p->token_bytes;
+    }
+    for (int64_t i = 0; i < fresh_n; ++i) {
+        s->blocks.push_back(got[(refetch ? 1 : 0) + i]);
+        s->img_tok.push_back(0);
+        s->hot_count += 1;
+    }
+    s->T += n;
+    s->last_use = ++p->clock;
+    p->lru_in(sid);
+    s->appended_recorded = !p->host_only;
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_appended += static_cast<int64_t>(n) * p->token_bytes;
+    p->stats.appends += 1;
+    return KV_OK;
+}
+
+// Resume with residency: only blocks no longer hot are fetched (misses);
+// the rest are hits.
+static int lru_resume(kv_pool *p, int32_t sid, cudaStream_t st) {
+    Session *s = &p->sessions[sid];
+    std::vector<int32_t> missing;
+    for (size_t j = 0; j < s->blocks.size(); ++j)
+        if (s->blocks[j] < 0) missing.push_back(static_cast<int32_t>(j));
+    const int64_t need = static_cast<int64_t>(missing.size());
+    std::vector<Victim> vic;
+    if (!p->plan_evict(need, {sid}, vic))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "no block can be evicted for the resume");
+    const std::vector<int32_t> got = p->peek_alloc(need, vic);
+    std::vector<int32_t> row(s->blocks);
+    std::vector<kvt::BlockJob> jobs;
+    int64_t fetched = 0;
+    for (int64_t i = 0; i < need; ++i) {
+        const int32_t j = missing[i];
+        row[j] = got[i];
+        jobs.push_back(p->job_for(sid, j, got[i], 0, p->tokens_in_block(*s, j)));
+        fetched += p->tokens_in_block(*s, j);
+    }
+
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    int rc = ensure_event(p, &s->ready);
+    if (!rc) rc = p->evict_device(vic, st);
+    if (!rc) rc = p->run_jobs(jobs, false, st);
+    if (!rc && need > 0) rc = p->write_table(sid, row.data(), 0, static_cast<int64_t>(row.size()), st);
+    if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
+    if (rc) return rc;
+
+    p->evict_commit(vic);
+    p->free_list.resize(p->free_list.size() - need);
+    p->lru_out(sid);
+    s->blocks = row;
+    s->hot_count += need;
+    s->state = KV_SESSION_ACTIVE;
+    s->last_use = ++p->clock;
+    p->lru_in(sid);
+    s->ready_recorded = !p->host_only;
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_unpacked += fetched * p->token_bytes;
+    p->stats.resume_blocks_hit += static_cast<int64_t>(s->blocks.size()) - need;
+    p->stats.resume_blocks_missed += need;
+    p->stats.resumes += 1;
+    return KV_OK;
+}
+
+// Before a decode step: bring back any block of the batch's sessions that was
+// evicted (no pinning: under pressure even active blocks spill), then stamp
+// all of them with one new recency time.
+static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStream_t st) {
+    std::vector<int32_t> uniq;
+    for (int32_t i = 0; i < B; ++i)
+        if (std::find(uniq.begin(), uniq.end(), sids[i]) == uniq.end()) uniq.push_back(sids[i]);
+    std::vector<std::vector<int32_t>> miss(uniq.size());
+    int64_t need = 0;
+    for (size_t u = 0; u < uniq.size(); ++u) {
+        const Session &s = p->sessions[uniq[u]];
+        for (size_t j = 0; j < s.blocks.size(); ++j)
+            if (s.blocks[j] < 0) miss[u].push_back(static_cast<int32_t>(j));
+        need += static_cast<int64_t>(miss[u].size());
+    }
+    std::vector<Victim> vic;
+    if (!p->plan_evict(need, uniq, vic))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "the batch's blocks do not fit in the hot pool");
+    const std::vector<int32_t> got = p->peek_alloc(need, vic);
+    std::vector<std::vector<int32_t>> rows(uniq.size());
+    std::vector<kvt::BlockJob> jobs;
+    int64_t k = 0, fetched = 0;
+    for (size_t u = 0; u < uniq.size(); ++u) {
+        const Session &s = p->sessions[uniq[u]];
+        rows[u] = s.blocks;
+        for (int32_t j : miss[u]) {
+            rows[u][j] = got[k];
+            jobs.push_back(p->job_for(uniq[u], j, got[k], 0, p->tokens_in_block(s, j)));
+            fetched += p->tokens_in_block(s, j);
+            ++k;
+        }
+    }
+    int rc = p->evict_device(vic, st);
+    if (!rc) rc = p->run_jobs(jobs, false, st);
+    for (size_t u = 0; !rc && u < uniq.size(); ++u)
+        if (!miss[u].empty())
+            rc = p->write_table(uniq[u], rows[u].data(), 0, static_cast<int64_t>(rows[u].size()), st);
+    if (rc) return rc;
+
+    p->evict_commit(vic);
+    p->free_list.resize(p->free_list.size() - need);
+    const uint64_t stamp = ++p->clock;
+    for (size_t u = 0; u < uniq.size(); ++u) {
+        Session &s = p->sessions[uniq[u]];
+        p->lru_out(uniq[u]);
+        s.blocks = rows[u];
+        s.hot_count += static_cast<int64_t>(miss[u].size());
+        s.last_use = stamp;
+        p->lru_in(uniq[u]);
+    }
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_unpacked += fetched * p->token_bytes;
+    return KV_OK;
+}
+
 int session_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_t n,
                    kv_stream_t stream_) {
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     Session *s = p->session(sid);
     if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    if (p->lru) return lru_append(p, sid, k, v, n, st);
     if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "append to a paused session");
     if (n < 1) return fail(KV_ERR_INVALID_ARG, "n must be >= 1");
     if (!p->host_only && (!k || !v)) return fail(KV_ERR_INVALID_ARG, "null k or v");
@@ -497,6 +816,11 @@ int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
     Session *s = p->session(sid);
     if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
     if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "pause of a session that is not active");
+    if (p->lru) {   // write-on-evict: nothing moves now; the blocks age in LRU order
+        s->state = KV_SESSION_PAUSED;
+        p->stats.pauses += 1;
+        return KV_OK;
+    }
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     DeviceGuard dg(p->cfg.device, !p->host_only);
 
@@ -545,6 +869,7 @@ int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
     Session *s = p->session(sid);
     if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
     if (s->state != KV_SESSION_PAUSED) return fail(KV_ERR_BAD_STATE, "resume of a session that is not paused");
+    if (p->lru) return lru_resume(p, sid, reinterpret_cast<cudaStream_t>(stream_));
     const int bt = p->cfg.block_tokens;
     const int64_t need = (s->T + bt - 1) / bt;
     if (need > static_cast<int64_t>(p->free_list.size()))
@@ -591,7 +916,7 @@ int session_info(kv_pool *p, int32_t sid, kv_session_info *out) {
     Session *s = p->session(sid);
     if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
     out->state = s->state;
-    out->num_blocks = static_cast<int32_t>(s->blocks.size());
+    out->num_blocks = static_cast<int32_t>(p->lru ? s->hot_count : static_cast<int64_t>(s->blocks.size()));
     out->tokens = s->T;
     out->capacity = s->cap;
     out->cold_valid = s->cold_valid;
@@ -612,8 +937,10 @@ int session_block_table(kv_pool *p, int32_t sid, int32_t *host_row, int32_t cap,
 int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
                          int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream_) {
     if (!p || !sids || B < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
-    if (p->host_only) return fail(KV_ERR_BAD_STATE, "batch tables on a host-logic-only pool");
-    if (!block_tables || !seq_lens || max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
+    if (p->host_only && !p->lru)
+        return fail(KV_ERR_BAD_STATE, "batch tables on a host-logic-only pool");
+    if (!p->host_only && (!block_tables || !seq_lens)) return fail(KV_ERR_INVALID_ARG, "null output");
+    if (max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "max_blocks must be >= 1");
     for (int32_t i = 0; i < B; ++i) {
         Session *s = p->session(sids[i]);
         if (!s) return fail(KV_ERR_INVALID_ARG, "no such session in batch");
@@ -624,6 +951,10 @@ int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *bl
     }
     DeviceGuard dg(p->cfg.device, true);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    if (p->lru) {
+        int rc = lru_fetch_batch(p, sids, B, st);
+        if (rc || p->host_only) return rc;   // host-logic pools: bookkeeping only
+    }
     for (int32_t r0 = 0; r0 < B; r0 += kvt::kGatherMax) {
         kvt::GatherArgs a;
         a.arena = p->d_tables;

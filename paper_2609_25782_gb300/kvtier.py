@@ -25,6 +25,7 @@ KV_ERR_CUDA = -5
 KV_ERR_DEVICE_CHECK = -6
 KV_SESSION_FREE, KV_SESSION_ACTIVE, KV_SESSION_PAUSED = 0, 1, 2
 KV_POOL_HOST_LOGIC_ONLY = 1
+KV_POOL_LRU_RESIDENCY = 2
 
 _ERR_NAMES = {v: k for k, v in globals().items() if k.startswith("KV_ERR_")}
 
@@ -65,7 +66,8 @@ class kv_session_info(C.Structure):
 class kv_pool_stats(C.Structure):
     _fields_ = [(n, C.c_int64) for n in (
         "free_blocks", "used_blocks", "cold_bytes_used", "bytes_unpacked", "bytes_packed",
-        "bytes_appended", "resumes", "pauses", "appends", "decodes")]
+        "bytes_appended", "resumes", "pauses", "appends", "decodes", "blocks_evicted",
+        "resume_blocks_hit", "resume_blocks_missed")]
 
 
 class KVError(RuntimeError):

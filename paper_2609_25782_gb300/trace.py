@@ -20,6 +20,7 @@ decides what to call and when.
 """
 from __future__ import annotations
 
+import dataclasses
 import heapq
 import math
 from dataclasses import dataclass, field
@@ -47,6 +48,7 @@ class TraceConfig:
     num_kv_heads: int = 4
     block_tokens: int = 16
     seed: int = 0
+    lru: bool = False                # block residency with LRU write-on-evict
 
 
 @dataclass
@@ -143,13 +145,16 @@ class TraceDriver:
         cfg = self.cfg
         now = k * cfg.dt_s
         tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
-        # 1. sessions whose burst ended last step pause (pack new tokens, free blocks)
-        if self.retire and self.gpu and self.last_decode_ev is not None:
+        # 1. sessions whose burst ended last step pause. Simple mode packs their
+        # new tokens and frees the blocks; residency mode moves nothing (the
+        # blocks age until evicted). Migrations may touch blocks the last
+        # decode step read, so they wait for it.
+        if self.gpu and self.last_decode_ev is not None and (self.retire or cfg.lru):
             self.mstream.wait_event(self.last_decode_ev)
         for i in self.retire:
             sid = self.sids[i]
             info = kvtier.session_info(self.pool, sid)
-            nbytes = (info.tokens - info.cold_valid) * tok_bytes
+            nbytes = 0 if cfg.lru else (info.tokens - info.cold_valid) * tok_bytes
             self._record_mig("pack", lambda: kvtier.session_pause(
                 self.pool, sid, self.mstream if self.gpu else None), nbytes)
             self.active.remove(i)
@@ -165,9 +170,13 @@ class TraceDriver:
                and self.queue[0][0] <= now):
             _, i = heapq.heappop(self.queue)
             sid = self.sids[i]
-            info = kvtier.session_info(self.pool, sid)
+            before = kvtier.kv_pool_get_stats(self.pool)["bytes_unpacked"]
             self._record_mig("unpack", lambda: kvtier.session_resume(
-                self.pool, sid, self.mstream if self.gpu else None), info.tokens * tok_bytes)
+                self.pool, sid, self.mstream if self.gpu else None), 0)
+            fetched = kvtier.kv_pool_get_stats(self.pool)["bytes_unpacked"] - before
+            if self.gpu:
+                kind, a, b, _ = self.mig_events[-1]
+                self.mig_events[-1] = (kind, a, b, fetched)
             n_ctx = self.trace[i].appends[self.turn[i]]
             self._append(i, n_ctx, self.mstream if self.gpu else None)
             self.counts["turn_tokens"] += n_ctx
@@ -193,8 +202,10 @@ class TraceDriver:
             self.counts["appended_tokens"] += len(members)
             blocks = sum(-(-self.tokens[i] // cfg.block_tokens) for i in self.active + self.joining)
             self.peak_blocks = max(self.peak_blocks, blocks)
+            sids = [self.sids[i] for i in members]
+            if not self.gpu and cfg.lru:     # recency and spilled-block fetches
+                kvtier.kv_pool_batch_tables(self.pool, sids, None, 1 << 20, None, None)
             if self.gpu:
-                sids = [self.sids[i] for i in members]
                 B = len(sids)
                 kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
                                             self.seq_lens, self.dstream)
@@ -221,25 +232,33 @@ class TraceDriver:
             self.step(k)
 
 
-def plan(cfg: TraceConfig, trace: list[SessionTrace]) -> dict:
+def plan(cfg: TraceConfig, trace: list[SessionTrace], hot_blocks: int | None = None) -> dict:
     """Dry run on a host-logic-only pool: per-session capacity and peak hot
-    blocks needed by the real run (the schedule does not depend on timing)."""
+    blocks needed by the real run (the schedule does not depend on timing).
+    With cfg.lru and hot_blocks, the dry run uses a residency-mode pool of
+    that size and its statistics are those the real run must reproduce."""
+    lru = cfg.lru and hot_blocks is not None
+    if cfg.lru and not lru:
+        cfg = dataclasses.replace(cfg, lru=False)
     tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
     big = cfg.sessions * (1 << 22) * tok_bytes    # host-logic pool: nothing is allocated
     c = kvtier.make_config(num_layers=cfg.layers, num_q_heads=cfg.num_q_heads,
                            num_kv_heads=cfg.num_kv_heads, block_tokens=cfg.block_tokens,
                            max_sessions=cfg.sessions, max_batch=cfg.active_cap,
-                           max_context=1 << 22, num_hot_blocks=300000,
-                           cold_bytes=big, flags=kvtier.KV_POOL_HOST_LOGIC_ONLY)
+                           max_context=1 << 22,
+                           num_hot_blocks=hot_blocks if lru else 300000, cold_bytes=big,
+                           flags=kvtier.KV_POOL_HOST_LOGIC_ONLY |
+                           (kvtier.KV_POOL_LRU_RESIDENCY if lru else 0))
     pool = kvtier.kv_pool_create(c)
     try:
         for t in trace:
             kvtier.session_create_paused(pool, 1 << 22, t.t0)
         d = TraceDriver(cfg, pool, trace, gpu=False)
         d.run()
+        stats = kvtier.kv_pool_get_stats(pool)
     finally:
         kvtier.kv_pool_destroy(pool)
     caps = [int(x) for x in d.peak_tokens]
-    return {"caps": caps, "peak_blocks": int(d.peak_blocks), "counts": d.counts,
+    return {"caps": caps, "peak_blocks": int(d.peak_blocks), "counts": d.counts, "stats": stats,
             "cold_bytes": int(sum(-(-(cap * tok_bytes) // 256) * 256 for cap in caps)),
             "max_context": int(max(caps))}

@@ -1,0 +1,141 @@
+"""Residency mode (LRU, write-on-evict) on the GPU: data, not just decisions.
+
+A random sequence of appends, pauses, resumes and decode batches runs on a
+small pool under pressure, with the residency oracle in lock step (it fixes
+which blocks are hot and which tokens each image holds). At every batch the
+decode output is checked against the attention oracle; at the end every hot
+block and every image prefix must hold the generator's values bit for bit.
+"""
+import math
+import random
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from oracle.residency import NoHotBlocks, ResidencyOracle
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+
+
+def bits(t):
+    return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def test_residency_random_sequence(cuda_dev):
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool, kvtier
+
+    L, Hq, Hkv, D, bt, nb, seed = 2, 32, 4, 128, 16, 40, 8
+    cap = 600
+    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=10 * cap * pool_token_bytes(L, Hkv),
+                max_sessions=10, max_batch=L * 4, max_context=cap, alloc_seed=seed,
+                lru_residency=True)
+    o = ResidencyOracle(nb, bt, seed=seed, token_bytes=pool.token_bytes)
+    rnd = random.Random(seed)
+    st = torch.cuda.Stream()
+    live, T = [], {}
+    q = synth.queries_torch(seed, range(4), range(L), Hq, D, cuda_dev)
+    mb = -(-cap // bt)
+    tables = torch.empty(4, mb, dtype=torch.int32, device=cuda_dev)
+    slens = torch.empty(4, dtype=torch.int32, device=cuda_dev)
+    checked = 0
+    for step in range(260):
+        r = rnd.random()
+        if r < 0.1 and len(live) < 8:
+            if rnd.random() < 0.5:
+                n0 = rnd.randint(20, 200)
+                sid = pool.session_create_paused(cap, n0)
+                synth.fill_image_torch(pool.image(sid), seed, sid, L, Hkv, D, n0)
+                o.create_paused(sid, cap, n0)
+                T[sid] = n0
+            else:
+                sid = pool.session_create(cap)
+                o.create(sid, cap)
+                T[sid] = 0
+            live.append(sid)
+            continue
+        if not live:
+            continue
+        sid = rnd.choice(live)
+        if o.s[sid].state == "paused":
+            try:
+                o.resume(sid)
+            except NoHotBlocks:
+                with pytest.raises(kvtier.KVError):
+                    pool.session_resume(sid, st)
+                continue
+            pool.session_resume(sid, st)
+        elif r < 0.55:
+            n = rnd.randint(1, 40)
+            if T[sid] + n > cap:
+                continue
+            try:
+                o.append(sid, n)
+            except NoHotBlocks:
+                continue
+            k, v = synth.kv_logical_torch(seed, sid, range(L), Hkv, D, T[sid], T[sid] + n, cuda_dev)
+            pool.session_append(sid, k.permute(0, 2, 1, 3).contiguous(),
+                                v.permute(0, 2, 1, 3).contiguous(), st)
+            T[sid] += n
+        elif r < 0.7:
+            o.pause(sid)
+            pool.session_pause(sid, st)
+        else:
+            batch = [x for x in live if o.s[x].state == "active" and T[x] > 0]
+            batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 4)))
+            if not batch:
+                continue
+            try:
+                o.batch(batch)
+            except NoHotBlocks:
+                continue
+            pool.batch_tables(batch, tables, mb, slens, st)
+            out = torch.empty(L, len(batch), Hq, D, dtype=torch.float32, device=cuda_dev)
+            with torch.cuda.stream(st):
+                pool.decode_attention(-1, q[:, :len(batch)].contiguous(), tables, slens, len(batch),
+                                      mb, 1 / math.sqrt(D), out, st)
+            torch.cuda.synchronize()
+            rows = np.full((len(batch), mb), -1, dtype=np.int32)
+            for i, x in enumerate(batch):
+                rows[i, :len(o.row(x))] = o.row(x)
+            lens = [T[x] for x in batch]
+            hot = synth.hot_pool_np(seed, batch, lens, rows, nb, L, Hkv, D, bt)
+            ref = oracle.paged_decode(hot, bits(q[:, :len(batch)]), rows, lens, 1 / math.sqrt(D), Hq)
+            got = out.double().cpu().numpy()
+            assert np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref))) <= TOL
+            checked += 1
+        assert pool.session_block_table(sid) == o.row(sid)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    stats = pool.stats()
+    for key in ("bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
+                "resume_blocks_missed"):
+        assert stats[key] == o.stats[key], key
+    assert stats["blocks_evicted"] > 10 and checked > 10
+    hv = pool.hot_view()
+    for sid in live:
+        s = o.s[sid]
+        k, v = synth.session_kv_np(seed, sid, range(L), Hkv, D, s.T)
+        img = bits(pool.image(sid))
+        for j, slot in enumerate(s.slots):
+            n = min(bt, s.T - j * bt)
+            if slot >= 0:                     # hot copy: the whole block
+                hb = bits(hv[slot])
+                assert np.array_equal(hb[:, 0, :, :n], k[:, :, j * bt:j * bt + n])
+                assert np.array_equal(hb[:, 1, :, :n], v[:, :, j * bt:j * bt + n])
+            m = s.img[j]                       # cold copy: the tokens written so far
+            assert np.array_equal(img[:, 0, :, j * bt:j * bt + m], k[:, :, j * bt:j * bt + m])
+            assert np.array_equal(img[:, 1, :, j * bt:j * bt + m], v[:, :, j * bt:j * bt + m])
+            if slot < 0:
+                assert m == n
+    pool.close()
+
+
+def pool_token_bytes(L, Hkv):
+    return L * 2 * Hkv * 128 * 2

@@ -1,0 +1,240 @@
+"""Block residency (LRU, write-on-evict) on the host, without a GPU.
+
+First the oracle's restatement of the policy is pinned to properties the
+paper states and to a scenario worked by hand; then the library's
+bookkeeping (a host-logic-only pool in residency mode) is compared with the
+oracle decision by decision on random operation sequences under pressure.
+"""
+import random
+
+import pytest
+
+import oracle
+from oracle.residency import NoHotBlocks, ResidencyOracle
+
+BT, TB = 16, 1000          # block tokens; bytes per token (any constant)
+
+
+def pack_tokens(o):
+    """token -> number of times it was written to the cold tier"""
+    cnt = {}
+    for kind, sid, j, slot, t0, t1 in o.log:
+        if kind == "pack":
+            for t in range(j * BT + t0, j * BT + t1):
+                cnt[(sid, t)] = cnt.get((sid, t), 0) + 1
+    return cnt
+
+
+def test_hand_worked_eviction_scenario():
+    o = ResidencyOracle(6, BT, seed=3, token_bytes=TB)
+    start = list(o.fl.contents())
+    o.create(0, 1000)
+    o.append(0, 40)            # A: 3 blocks, time 1
+    o.create(1, 1000)
+    o.append(1, 32)            # B: 2 blocks, time 2
+    assert o.fl.n == 1
+    a_slots = o.row(0)
+    assert a_slots == [start[5], start[4], start[3]]     # popped from the end
+    o.pause(0)
+    o.create(2, 1000)
+    o.append(2, 40)            # C needs 3 blocks: 1 free + A's blocks 0 and 1 (A least recent)
+    assert o.row(0) == [-1, -1, a_slots[2]]
+    assert o.stats["blocks_evicted"] == 2
+    assert o.stats["bytes_packed"] == 32 * TB             # two full blocks, written once
+    o.resume(0)                # A's blocks 0,1 missing: evict B's (LRU among B, C), hit = 1
+    assert o.stats["resume_blocks_hit"] == 1 and o.stats["resume_blocks_missed"] == 2
+    assert o.row(1) == [-1, -1]
+    assert o.stats["bytes_packed"] == 64 * TB             # + B's 32 tokens
+    assert o.stats["bytes_unpacked"] == 32 * TB           # A's two blocks back
+    o.pause(0)
+    o.resume(0)                # nothing evicted since: all hits, nothing moves
+    assert o.stats["resume_blocks_hit"] == 4 and o.stats["bytes_unpacked"] == 32 * TB
+
+
+def test_each_token_written_at_most_once():
+    rnd = random.Random(5)
+    o = ResidencyOracle(10, BT, seed=1, token_bytes=TB)
+    for sid in range(4):
+        o.create(sid, 10_000)
+    for _ in range(400):
+        sid = rnd.randrange(4)
+        s = o.s[sid]
+        try:
+            if s.state == "active":
+                if rnd.random() < 0.7:
+                    o.append(sid, rnd.randint(1, 30))
+                else:
+                    o.pause(sid)
+            else:
+                o.resume(sid)
+        except NoHotBlocks:
+            pass
+    cnt = pack_tokens(o)
+    assert cnt and max(cnt.values()) == 1
+    total = sum(s.T for s in o.s.values())
+    assert o.stats["bytes_packed"] <= total * TB
+
+
+def test_no_pressure_no_eviction_full_hits():
+    o = ResidencyOracle(100, BT, seed=2, token_bytes=TB)
+    for sid in range(3):
+        o.create(sid, 1000)
+        o.append(sid, 100)
+        o.pause(sid)
+    for sid in range(3):
+        o.resume(sid)
+    assert o.stats["blocks_evicted"] == 0 and o.stats["bytes_packed"] == 0
+    assert o.stats["resume_blocks_missed"] == 0 and o.stats["resume_blocks_hit"] == 21
+
+
+def test_recency_keeps_the_active_set_hot():
+    """Batched every step, the active sessions are always the most recent:
+    with room for them, only idle sessions' blocks are evicted."""
+    o = ResidencyOracle(40, BT, seed=4, token_bytes=TB)
+    active, idle = [0, 1, 2], [3, 4, 5, 6]
+    for sid in active + idle:
+        o.create(sid, 10_000)
+    for sid in idle:
+        o.append(sid, 64)
+        o.pause(sid)
+    for sid in active:
+        o.append(sid, 100)
+    for step in range(100):    # the active set grows to 3 x 13 = 39 of 40 blocks
+        o.batch(active)
+        for sid in active:
+            o.append(sid, 1)
+        assert all(slot >= 0 for sid in active for slot in o.row(sid))
+    assert o.stats["blocks_evicted"] > 0
+    evicted_active = [l for l in o.log if l[0] == "pack" and l[1] in active]
+    assert not evicted_active
+
+
+def test_no_pinning_spills_instead_of_failing():
+    o = ResidencyOracle(8, BT, seed=6, token_bytes=TB)
+    o.create(0, 1000)
+    o.append(0, 64)            # 4 blocks
+    o.create(1, 1000)
+    o.append(1, 64)            # 4 blocks: pool full, both active
+    o.append(0, 16)            # needs one more: session 1 (active, older) spills a block
+    assert o.row(1)[0] == -1
+    o.batch([1])               # bringing it back evicts session 0's oldest block
+    assert all(x >= 0 for x in o.row(1)) and o.row(0)[0] == -1
+    with pytest.raises(NoHotBlocks):
+        o.batch([0, 1])        # 9 blocks can never fit in 8
+
+
+# ------------------------------------------------ library vs oracle
+
+@pytest.fixture(scope="module")
+def kv():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import kvtier
+    return kvtier
+
+
+def lib_pool(kv, nb, seed):
+    cfg = kv.make_config(num_layers=1, num_hot_blocks=nb, block_tokens=BT, alloc_seed=seed,
+                         max_sessions=8, max_context=4096, max_batch=8,
+                         cold_bytes=8 * 4096 * 2 * 4 * 128 * 2,
+                         flags=kv.KV_POOL_HOST_LOGIC_ONLY | kv.KV_POOL_LRU_RESIDENCY)
+    return kv.kv_pool_create(cfg), kv.kv_token_bytes(cfg)
+
+
+def compare(kv, pool, o, sids):
+    assert kv.kv_pool_free_list(pool) == list(o.fl.contents())
+    for sid in sids:
+        assert kv.session_block_table(pool, sid) == o.row(sid)
+        info = kv.session_info(pool, sid)
+        assert info.tokens == o.s[sid].T
+        assert info.state == (kv.KV_SESSION_ACTIVE if o.s[sid].state == "active"
+                              else kv.KV_SESSION_PAUSED)
+    st = kv.kv_pool_get_stats(pool)
+    for k, v in o.stats.items():
+        assert st[k] == v, k
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+def test_library_matches_oracle_on_random_sequences(kv, seed):
+    rnd = random.Random(seed)
+    nb = 14
+    pool, tb = lib_pool(kv, nb, seed)
+    o = ResidencyOracle(nb, BT, seed=seed, token_bytes=tb)
+    live = []
+    fails = 0
+    for step in range(500):
+        r = rnd.random()
+        try:
+            if r < 0.08 and len(live) < 6:
+                if rnd.random() < 0.5:
+                    T = rnd.randint(1, 90)
+                    sid = kv.session_create_paused(pool, 400, T)
+                    o.create_paused(sid, 400, T)
+                else:
+                    sid = kv.session_create(pool, 400)
+                    o.create(sid, 400)
+                live.append(sid)
+            elif r < 0.12 and live:
+                sid = rnd.choice(live)
+                kv.session_destroy(pool, sid)
+                o.destroy(sid)
+                live.remove(sid)
+            elif r < 0.14:
+                s = rnd.randrange(1 << 30)
+                kv.kv_pool_shuffle_free(pool, s)
+                o.shuffle(s)
+            elif live:
+                sid = rnd.choice(live)
+                state = o.s[sid].state
+                if state == "paused":
+                    exp = None
+                    try:
+                        o.resume(sid)
+                    except NoHotBlocks:
+                        exp = kv.KV_ERR_NO_HOT_BLOCKS
+                    try:
+                        kv.session_resume(pool, sid)
+                        assert exp is None
+                    except kv.KVError as e:
+                        assert e.code == exp
+                        fails += 1
+                elif r < 0.6:
+                    n = rnd.randint(1, 24)
+                    if o.s[sid].T + n > 400:
+                        continue
+                    exp = None
+                    try:
+                        o.append(sid, n)
+                    except NoHotBlocks:
+                        exp = kv.KV_ERR_NO_HOT_BLOCKS
+                    try:
+                        kv.session_append(pool, sid, None, None, n, None)
+                        assert exp is None
+                    except kv.KVError as e:
+                        assert e.code == exp
+                        fails += 1
+                elif r < 0.75:
+                    o.pause(sid)
+                    kv.session_pause(pool, sid, None)
+                else:
+                    batch = [x for x in live if o.s[x].state == "active" and o.s[x].T > 0]
+                    batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 3)))
+                    if not batch:
+                        continue
+                    exp = None
+                    try:
+                        o.batch(batch)
+                    except NoHotBlocks:
+                        exp = kv.KV_ERR_NO_HOT_BLOCKS
+                    try:
+                        kv.kv_pool_batch_tables(pool, batch, None, 64, None)
+                        assert exp is None
+                    except kv.KVError as e:
+                        assert e.code == exp
+                        fails += 1
+        finally:
+            pass
+        compare(kv, pool, o, live)
+    st = kv.kv_pool_get_stats(pool)
+    assert st["blocks_evicted"] > 20 and st["resume_blocks_missed"] > 0
+    kv.kv_pool_destroy(pool)
