@@ -54,9 +54,10 @@ def recorded_traffic():
     try:
         with open(os.path.join(ROOT, "profiles", "decode_split_kernel.traffic.json")) as f:
             rec = json.load(f)
-        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
-                return None
+        for path, sha in rec["sources_sha256"].items():
+            with open(os.path.join(ROOT, path), "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest() != sha:
+                    return None
         return int(rec["dram_bytes_per_launch"])
     except Exception:
         return None
@@ -482,10 +483,10 @@ def run_sweep(args):
         nb = max_tok // bt + 64
         Bmax = max(B for B, _ in pts)
         # workspace rows: the largest of layers x B x Hq x splits(T) over the points
-        need = max(L * B * HQ * max(16, -(-T // 512)) for B, T in pts)
+        need = max(L * B * HQ * -(-T // 2048) for B, T in pts)
         ctx = max(SWEEP_T)
         pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,
-                    max_sessions=4, max_batch=-(-need // (HQ * max(16, -(-ctx // 512)))),
+                    max_sessions=4, max_batch=-(-need // (HQ * -(-ctx // 2048))),
                     max_context=ctx, device=dev.index)
         # values: one synthetic session laid over the whole pool (finite N(0,1))
         synth.fill_hot_pool_torch(pool.hot, args.seed, [0], [nb * bt], [np.arange(nb)], L, HKV, D,

@@ -40,8 +40,10 @@ def build(force: bool = False, verbose: bool = False) -> str:
     cc = nvcc()
     out_dir = os.path.join(HERE, "_build")
     os.makedirs(out_dir, exist_ok=True)
+    # KVT_EXTRA_NVCC_FLAGS: extra -D tuning definitions for experiments
+    extra_flags = os.environ.get("KVT_EXTRA_NVCC_FLAGS", "").split()
     common = [cc, "-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", *ARCH,
-              "-I", os.path.join(HERE, "..", "include")]
+              "-I", os.path.join(HERE, "..", "include"), *extra_flags]
     procs, objs = [], []
     for src in SOURCES:
         obj = os.path.join(out_dir, src + ".o")

@@ -26,8 +26,15 @@
 namespace kvt {
 namespace {
 
-constexpr int kDecodeWarps = 4;
-constexpr int kStages = 3;                 // tiles in flight per warp
+#ifndef KVT_DECODE_WARPS
+#define KVT_DECODE_WARPS 4
+#endif
+#ifndef KVT_STAGES
+#define KVT_STAGES 2   // 4 warps x 2 x 8 KiB: 3 CTAs (24 tiles in flight) per SM
+#endif
+constexpr int kDecodeWarps = KVT_DECODE_WARPS;
+constexpr int kStages = KVT_STAGES;        // tiles in flight per warp
+constexpr int kCombineWarps = 4;
 constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
 constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
 constexpr int kDecodeSmem = kDecodeWarps * kStages * kTileBytes + 1024 + 256;
@@ -142,7 +149,7 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 // The four warps' states merge in shared memory in warp order; a one-split
 // session writes its normalised output, others write (m, l, acc) partials.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kDecodeWarps * 32, 2)
+__global__ void __launch_bounds__(kDecodeWarps * 32)
     decode_split_kernel(const __grid_constant__ CUtensorMap map, const DecodeArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -429,11 +436,11 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     const int64_t base = row * a.max_splits;
     const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml) + base;
     const float4 *po = reinterpret_cast<const float4 *>(a.part_o + base * kHeadDim) + lane;
-    __shared__ float s_m[kDecodeWarps], s_l[kDecodeWarps];
-    __shared__ float4 s_acc[kDecodeWarps][kHeadDim / 4];
+    __shared__ float s_m[kCombineWarps], s_l[kCombineWarps];
+    __shared__ float4 s_acc[kCombineWarps][kHeadDim / 4];
 
-    const int s0 = (warp * ns) / kDecodeWarps;
-    const int s1 = ((warp + 1) * ns) / kDecodeWarps;
+    const int s0 = (warp * ns) / kCombineWarps;
+    const int s1 = ((warp + 1) * ns) / kCombineWarps;
     float m = -INFINITY, lsum = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
@@ -459,11 +466,11 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     if (warp == 0) {
         float M = s_m[0];
 #pragma unroll
-        for (int w = 1; w < kDecodeWarps; ++w) M = fmaxf(M, s_m[w]);
+        for (int w = 1; w < kCombineWarps; ++w) M = fmaxf(M, s_m[w]);
         float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
         float l = 0.f;
 #pragma unroll
-        for (int w = 0; w < kDecodeWarps; ++w) {
+        for (int w = 0; w < kCombineWarps; ++w) {
             const float c = ex2(s_m[w] - M);       // an empty quarter has m = -inf: c = 0
             const float4 x = s_acc[w][lane];
             r.x += c * x.x;
@@ -672,7 +679,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStrea
 
     cudaLaunchConfig_t c2 = {};
     c2.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
-    c2.blockDim = dim3(kDecodeWarps * 32);
+    c2.blockDim = dim3(kCombineWarps * 32);
     c2.dynamicSmemBytes = 0;
     c2.stream = st;
     c2.attrs = attr;
