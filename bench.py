@@ -370,7 +370,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     from paper_2609_25782_gb300 import Pool, kvtier
     from paper_2609_25782_gb300 import trace as tr
     dev = torch.device("cuda", torch.cuda.current_device())
-    cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps)
+    cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps,
+                         admit_lead=args.trace_admit_lead)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -383,6 +384,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
                 max_sessions=cfg.sessions, max_batch=cfg.active_cap,
                 max_context=plan["max_context"], alloc_seed=cfg.seed, device=dev.index,
                 lru_residency=cfg.lru)
+    kvtier.kv_pool_set_migration_limit(pool.handle, args.trace_mig_ctas)
     for i, t in enumerate(trace):
         sid = pool.session_create_paused(plan["caps"][i], t.t0)
         synth.fill_image_torch(pool.image(sid), cfg.seed, sid, cfg.layers, cfg.num_kv_heads, D,
@@ -416,7 +418,10 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
     flags = pool.check_device()
-    steps_ms = sorted(a.elapsed_time(b) for a, b, _ in d.step_events)
+    step_t = [(a.elapsed_time(b), tok) for a, b, _, tok in d.step_events]
+    steps_ms = sorted(t for t, _ in step_t)
+    # per-step decode bandwidth: separates workload size from interference
+    step_gbs = sorted(tok * TOKEN_BYTES / (t * 1e-3) / 1e9 for t, tok in step_t)
     mig = {"unpack": [0.0, 0], "pack": [0.0, 0]}
     for kind, a, b, nbytes in d.mig_events:
         mig[kind][0] += a.elapsed_time(b)
@@ -429,10 +434,17 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     def pct(p):
         return steps_ms[min(len(steps_ms) - 1, int(round(p / 100 * (len(steps_ms) - 1))))]
 
-    extra = {}
+    from paper_2609_25782_gb300 import tiering_model
+    sim_s = cfg.steps * cfg.dt_s
+    model = tiering_model.from_trace(
+        cold_write_bytes=st["bytes_packed"], hot_read_bytes=d.counts["decode_tokens"] * TOKEN_BYTES,
+        cold_read_bytes=st["bytes_unpacked"], simulated_seconds=sim_s)
+    extra = {"model": {k: (round(v, 3) if isinstance(v, float) and v != float("inf") else
+                           (None if v == float("inf") else v)) for k, v in model.items()},
+             "simulated_s": sim_s}
     if cfg.lru:
         hit, miss = st["resume_blocks_hit"], st["resume_blocks_missed"]
-        extra = {"mode": "LRU block residency, write-on-evict", "hot_blocks": nb,
+        extra.update({"mode": "LRU block residency, write-on-evict", "hot_blocks": nb,
                  "hot_vs_simple_peak": lru_factor,
                  "resume_hit_rate": round(hit / max(1, hit + miss), 4),
                  "blocks_evicted": st["blocks_evicted"],
@@ -440,13 +452,16 @@ def run_trace(args, rank, lru_factor: float = 0.0):
                  "cold_read_gb": round(st["bytes_unpacked"] / 1e9, 2),
                  "matches_dry_run": all(st[k] == dry[k] for k in (
                      "bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
-                     "resume_blocks_missed", "resumes", "pauses"))}
+                     "resume_blocks_missed", "resumes", "pauses"))})
     return {
         **extra,
+        "admit_lead": cfg.admit_lead, "mig_ctas": args.trace_mig_ctas,
         "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
         "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
         "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2),
-        "mean_batch": round(sum(b for _, _, b in d.step_events) / max(1, len(d.step_events)), 2),
+        "mean_batch": round(sum(e[2] for e in d.step_events) / max(1, len(d.step_events)), 2),
+        "step_kv_gbs_p50": round(step_gbs[len(step_gbs) // 2], 1),
+        "step_kv_gbs_p1": round(step_gbs[len(step_gbs) // 100], 1),
         "resumes": st["resumes"], "pauses": st["pauses"],
         "unpack_gb": round(mig["unpack"][1] / 1e9, 2),
         "unpack_gbs": round(mig["unpack"][1] / max(1e-9, mig["unpack"][0] * 1e-3) / 1e9, 1),
@@ -651,6 +666,10 @@ def main():
     ap.add_argument("--mig-sessions", type=int, default=8)
     ap.add_argument("--mig-tokens", type=int, default=32768)
     ap.add_argument("--trace-steps", type=int, default=2000)
+    ap.add_argument("--trace-admit-lead", type=int, default=1,
+                    help="steps between a session's resume and its first decode step")
+    ap.add_argument("--trace-mig-ctas", type=int, default=0,
+                    help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--no-trace", action="store_true")
     ap.add_argument("--no-overlap", action="store_true",
                     help="launch every decode call fully serialised (no programmatic overlap)")

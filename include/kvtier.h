@@ -260,6 +260,13 @@ int kv_pool_get_stats(kv_pool *pool, kv_pool_stats *out);
  * non-zero value makes the call return KV_ERR_DEVICE_CHECK. */
 int kv_pool_check_device(kv_pool *pool, int32_t *flags);
 
+/* Cap the migration kernels (resume-unpack, pause-pack, evictions) at about
+ * max_ctas CTAs of 256 threads (rounded up to 8 per SM-sized unit), so that
+ * migrations running beside decode take a smaller share of HBM bandwidth
+ * (Section 3, data paths: eviction and resume overlap decode). 0 removes the
+ * cap (the default: 8 CTAs per SM). Affects later calls only. */
+int kv_pool_set_migration_limit(kv_pool *pool, int32_t max_ctas);
+
 /* Test hook: make the n-th following CUDA call of this pool fail (as a
  * CUDA error) so tests can check that failing calls change nothing;
  * n <= 0 disarms. */

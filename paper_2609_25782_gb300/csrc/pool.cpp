@@ -97,7 +97,15 @@ struct kv_pool {
     int32_t max_splits = 0;              // split bound for max_context
     int64_t part_rows = 0;               // decode workspace capacity (partial rows)
     int num_sms = 1;
+    int mig_ctas = 0;                    // cap on migration-kernel CTAs, 0 = none
     kvt::Shape shape{};
+
+    // SM budget handed to the migration kernels (8 CTAs per unit).
+    int mig_units() const {
+        if (mig_ctas <= 0) return num_sms;
+        const int u = (mig_ctas + 7) / 8;
+        return u < 1 ? 1 : u;
+    }
 
     std::vector<int32_t> free_list;      // top = back
     std::vector<int16_t> block_fence;    // fence slot of the pack that freed it, or -1
@@ -316,7 +324,7 @@ struct kv_pool {
             a.pad = 0;
             std::copy(jobs.begin() + i, jobs.begin() + i + a.n, a.job);
             int rc = cuda(pack ? "pack launch" : "unpack launch",
-                          [&] { return kvt::launch_block_jobs(a, pack, num_sms, st); });
+                          [&] { return kvt::launch_block_jobs(a, pack, mig_units(), st); });
             if (rc) return rc;
         }
         return KV_OK;
@@ -839,7 +847,7 @@ int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
         kvt::MigArgs m = p->mig_args(sid, *s);
         m.t_begin = static_cast<int32_t>(t0);
         m.t_end = static_cast<int32_t>(t1);
-        rc = p->cuda("pack launch", [&] { return kvt::launch_pack(m, p->num_sms, st); });
+        rc = p->cuda("pack launch", [&] { return kvt::launch_pack(m, p->mig_units(), st); });
     }
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(p->fences[f].ev, st); });
     if (rc) return rc;
@@ -886,7 +894,7 @@ int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
         kvt::MigArgs m = p->mig_args(sid, *s);
         m.t_begin = 0;
         m.t_end = static_cast<int32_t>(s->T);
-        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->num_sms, st); });
+        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->mig_units(), st); });
     }
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
     if (rc) return rc;
@@ -1009,6 +1017,12 @@ int kv_pool_check_device(kv_pool *p, int32_t *flags) {
     if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_err, 0, 4); });
     if (rc) return rc;
     if (*flags) return fail(KV_ERR_DEVICE_CHECK, "a kernel bounds check fired (flags " + std::to_string(*flags) + ")");
+    return KV_OK;
+}
+
+int kv_pool_set_migration_limit(kv_pool *p, int32_t max_ctas) {
+    if (!p || max_ctas < 0) return fail(KV_ERR_INVALID_ARG, "bad argument");
+    p->mig_ctas = max_ctas;
     return KV_OK;
 }
 

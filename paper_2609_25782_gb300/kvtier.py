@@ -37,7 +37,7 @@ EXPORTS = [
     "session_info", "session_block_table", "kv_pool_batch_tables", "kv_pool_shuffle_free",
     "kv_pool_free_list", "kv_pool_get_stats", "kv_pool_check_device",
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
-    "decode_attention_ex",
+    "decode_attention_ex", "kv_pool_set_migration_limit",
 ]
 
 KV_DECODE_OVERLAP_PREVIOUS = 1
@@ -104,6 +104,7 @@ def _load():
         "kv_pool_get_stats": [p, C.POINTER(kv_pool_stats)],
         "kv_pool_check_device": [p, C.POINTER(i32)],
         "kv_pool_inject_cuda_failure": [p, i32],
+        "kv_pool_set_migration_limit": [p, i32],
         "kv_last_error": [],
         "decode_attention_noalloc": [C.POINTER(kv_pool_config), i32, p, p, p, i32, i32,
                                      C.c_float, p, p],
@@ -262,6 +263,10 @@ def kv_pool_check_device(pool: int) -> int:
     if rc not in (KV_OK, KV_ERR_DEVICE_CHECK):
         _check(rc, "kv_pool_check_device")
     return flags.value
+
+
+def kv_pool_set_migration_limit(pool: int, max_ctas: int) -> None:
+    _check(lib.kv_pool_set_migration_limit(pool, max_ctas), "kv_pool_set_migration_limit")
 
 
 def kv_pool_inject_cuda_failure(pool: int, n: int) -> None:

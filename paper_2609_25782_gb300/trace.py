@@ -49,6 +49,7 @@ class TraceConfig:
     block_tokens: int = 16
     seed: int = 0
     lru: bool = False                # block residency with LRU write-on-evict
+    admit_lead: int = 1              # steps between a resume and the session's first decode
 
 
 @dataclass
@@ -101,7 +102,7 @@ class TraceDriver:
         self.queue = [(t.first_ready_s, i) for i, t in enumerate(trace)]
         heapq.heapify(self.queue)
         self.active: list[int] = []          # decoding this step
-        self.joining: list[int] = []         # admitted this step, decode from the next
+        self.joining: list[tuple[int, int]] = []   # (first decode step, session) admitted
         self.retire: list[int] = []
         self.peak_tokens = list(self.tokens)
         self.peak_blocks = 0
@@ -162,9 +163,9 @@ class TraceDriver:
             self.turn[i] += 1
             self.counts["pauses"] += 1
         self.retire = []
-        # sessions admitted last step join the batch now
-        self.active.extend(self.joining)
-        self.joining = []
+        # sessions whose admission lead has passed join the batch now
+        self.active.extend(i for j, i in self.joining if j <= k)
+        self.joining = [(j, i) for j, i in self.joining if j > k]
         # 2. admit ready sessions while below the cap (resume + turn context)
         while (len(self.active) + len(self.joining) < cfg.active_cap and self.queue
                and self.queue[0][0] <= now):
@@ -185,7 +186,7 @@ class TraceDriver:
                 ev = self._torch.cuda.Event()
                 ev.record(self.mstream)
                 self.admit_ev[i] = ev
-            self.joining.append(i)
+            self.joining.append((k + max(1, cfg.admit_lead), i))
             self.counts["resumes"] += 1
         # 3. decode step for the active batch
         members = sorted(self.active)
@@ -200,7 +201,8 @@ class TraceDriver:
             for i in members:                 # this step's token (path 3)
                 self._append(i, 1, self.dstream if self.gpu else None)
             self.counts["appended_tokens"] += len(members)
-            blocks = sum(-(-self.tokens[i] // cfg.block_tokens) for i in self.active + self.joining)
+            blocks = sum(-(-self.tokens[i] // cfg.block_tokens)
+                         for i in self.active + [i for _, i in self.joining])
             self.peak_blocks = max(self.peak_blocks, blocks)
             sids = [self.sids[i] for i in members]
             if not self.gpu and cfg.lru:     # recency and spilled-block fetches
@@ -217,7 +219,7 @@ class TraceDriver:
                         kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 else 0, self.dstream)
                 end.record(self.dstream)
                 self.last_decode_ev = end
-                self.step_events.append((start, end, B))
+                self.step_events.append((start, end, B, sum(self.tokens[i] for i in members)))
                 if self.on_step is not None:
                     self.on_step(k, members)
             self.counts["decode_tokens"] += sum(self.tokens[i] for i in members)
