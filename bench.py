@@ -186,10 +186,19 @@ def run_decode(args, ws, rank):
     # `out`, so it may overlap its start with that call's end.
     ov = not args.no_overlap
 
-    def step():
+    def step_calls(st):
         for l in range(L):
-            pool.decode_attention(l, q[l], tables, lens_d, B2, max_blocks, scale, out[l], stream,
+            pool.decode_attention(l, q[l], tables, lens_d, B2, max_blocks, scale, out[l], st,
                                   overlap_previous=ov and l > 0)
+
+    graph = capture_graph(step_calls, stream) if args.graph else None
+
+    def step():
+        if graph is not None:
+            with torch.cuda.stream(stream):
+                graph.replay()
+        else:
+            step_calls(stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -215,50 +224,93 @@ def run_decode(args, ws, rank):
     total_ms = t0.elapsed_time(t1)
     launch_ms = total_ms / (args.steps * L)     # average decode call over the timed region
 
-    # end to end through the C ABI with host buffers
+    # End to end through the C ABI with host buffers: every step copies its
+    # Q, block tables and seq_lens from pinned host memory and reads its
+    # outputs back. Inputs and outputs are double-buffered so that step k+1's
+    # upload and step k's read-back run on a copy stream while step k decodes.
+    cs = torch.cuda.Stream(device=dev)
     q_h = torch.empty(q.shape, dtype=q.dtype).pin_memory()
     q_h.copy_(q.cpu())
     tab_h = torch.as_tensor(tables_h).pin_memory()
     len_h = torch.as_tensor(lens.astype(np.int32)).pin_memory()
-    out_h = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    q_d = torch.empty_like(q)
-    tab_d = torch.empty_like(tables)
-    len_d2 = torch.empty_like(lens_d)
+    out_h = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+    q_d = [torch.empty_like(q) for _ in range(2)]
+    tab_d = [torch.empty_like(tables) for _ in range(2)]
+    len_d = [torch.empty_like(lens_d) for _ in range(2)]
+    out_d = [torch.empty_like(out) for _ in range(2)]
+    up_done = [torch.cuda.Event() for _ in range(2)]
+    dec_done = [torch.cuda.Event() for _ in range(2)]
+    down_done = [torch.cuda.Event() for _ in range(2)]
+    for ev in up_done + dec_done + down_done:
+        ev.record(cs)
 
-    def e2e_step():
-        q_d.copy_(q_h, non_blocking=True)
-        tab_d.copy_(tab_h, non_blocking=True)
-        len_d2.copy_(len_h, non_blocking=True)
-        for l in range(L):
-            pool.decode_attention(l, q_d[l], tab_d, len_d2, B2, max_blocks, scale, out[l], stream,
-                                  overlap_previous=ov and l > 0)
-        out_h.copy_(out, non_blocking=True)
+    def upload(buf):
+        with torch.cuda.stream(cs):
+            cs.wait_event(dec_done[buf])          # the decode that read this buffer is done
+            q_d[buf].copy_(q_h, non_blocking=True)
+            tab_d[buf].copy_(tab_h, non_blocking=True)
+            len_d[buf].copy_(len_h, non_blocking=True)
+            up_done[buf].record(cs)
 
-    with torch.cuda.stream(stream):
-        for _ in range(max(1, args.warmup // 2)):
-            e2e_step()
+    def e2e_run(nsteps):
+        upload(0)
+        for k in range(nsteps):
+            buf = k % 2
+            if k + 1 < nsteps:
+                upload(buf ^ 1)
+            stream.wait_event(up_done[buf])
+            stream.wait_event(down_done[buf])     # this output buffer was read back
+            for l in range(L):
+                pool.decode_attention(l, q_d[buf][l], tab_d[buf], len_d[buf], B2, max_blocks,
+                                      scale, out_d[buf][l], stream, overlap_previous=ov and l > 0)
+            dec_done[buf].record(stream)
+            with torch.cuda.stream(cs):
+                cs.wait_event(dec_done[buf])
+                out_h[buf].copy_(out_d[buf], non_blocking=True)
+                down_done[buf].record(cs)
+        stream.wait_event(down_done[(nsteps - 1) % 2])
+
+    e2e_run(max(1, args.warmup // 2))
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     if ws > 1:
         dist.barrier()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(args.steps):
-            e2e_step()
-        e1.record(stream)
+    e0.record(stream)
+    cs.wait_event(e0)
+    e2e_run(args.steps)
+    e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     if ws > 1:
         dist.barrier()
 
     res = {
+        "graph": graph is not None,
         "total_ms": total_ms, "launch_ms": launch_ms, "kv_bytes": kv_bytes, "e2e_ms": e2e_ms,
         "launch_alg_bytes": launch_alg_bytes, "setup_s": setup_s, "clocks": clk.summary(),
         "h2d": q.numel() * 2 + tables.numel() * 4 + lens_d.numel() * 4,
         "d2h": out.numel() * 4, "pool": pool, "lens": lens, "tables": tables_h,
     }
     return res
+
+
+def capture_graph(calls, stream):
+    """One CUDA graph of `calls(capture_stream)` (the library's launches are
+    recorded like any other stream work), or None if capture fails."""
+    import torch
+    try:
+        with torch.cuda.stream(stream):
+            calls(stream)                      # warm the launch path outside capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            calls(torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        return g
+    except Exception as e:                     # report and fall back to direct launches
+        print(f"graph capture failed, launching directly: {e}", file=sys.stderr)
+        return None
 
 
 def run_migration(args, rank):
@@ -515,14 +567,22 @@ def run_sweep(args):
             q = synth.queries_torch(args.seed, range(B), range(L), HQ, D, dev).contiguous()
             out = torch.empty(L, B, HQ, D, dtype=torch.float32, device=dev)
             res = {"block_tokens": bt, "B": B, "T": T}
+            def per_layer(st):
+                for l in range(L):
+                    pool.decode_attention(l, q[l], tab, sl, B, tab.shape[1], scale, out[l], st,
+                                          overlap_previous=l > 0)
+
+            g = capture_graph(per_layer, stream) if args.graph else None
+            res["graph"] = g is not None
             for mode in ("per_layer", "all_layers"):
                 def step():
                     if mode == "all_layers":
                         pool.decode_attention(-1, q, tab, sl, B, tab.shape[1], scale, out, stream)
+                    elif g is not None:
+                        with torch.cuda.stream(stream):
+                            g.replay()
                     else:
-                        for l in range(L):
-                            pool.decode_attention(l, q[l], tab, sl, B, tab.shape[1], scale, out[l],
-                                                  stream, overlap_previous=l > 0)
+                        per_layer(stream)
                 kv = B * T * TOKEN_BYTES
                 reps = max(3, min(50, int(2e11 // kv)))
                 for _ in range(2):
@@ -538,7 +598,7 @@ def run_sweep(args):
                 gbs = kv / (ms * 1e-3) / 1e9
                 res[mode] = {"ms": round(ms, 4), "kv_gbs": round(gbs, 1), "frac": round(gbs / peak, 3)}
             points.append(res)
-            del q, out, tab, sl
+            del q, out, tab, sl, g
         flags = pool.check_device()
         if flags:
             raise RuntimeError(f"device check flags {flags} in the sweep")
@@ -671,6 +731,8 @@ def main():
     ap.add_argument("--trace-mig-ctas", type=int, default=0,
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--no-trace", action="store_true")
+    ap.add_argument("--graph", action=argparse.BooleanOptionalAction, default=True,
+                    help="replay the per-layer calls of a step from one CUDA graph")
     ap.add_argument("--no-overlap", action="store_true",
                     help="launch every decode call fully serialised (no programmatic overlap)")
     ap.add_argument("--sweep", action="store_true",
@@ -751,6 +813,7 @@ def main():
                 "workload": f"decode-attention step: {shape}, random physical blocks",
                 "tokens": int(np.sum(res["lens"])), "kv_gb_per_step": round(res["kv_bytes"] / 1e9, 2),
                 "launches_per_step": 2 * nl, "compute": "bf16 inputs, fp32 softmax/accumulate",
+                "cuda_graph": res["graph"],
                 "l2": f"inputs larger than L2 (KV per layer call {res['kv_bytes'] / nl / 1e9:.2f} GB)",
                 "parallelism": f"replicas x{ws} (sessions sharded, no collective)",
             },

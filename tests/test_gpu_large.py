@@ -101,12 +101,26 @@ def test_decode_full_size_bench_configuration(P, cuda_dev):
     len_d = torch.as_tensor(lens.astype(np.int32), device=cuda_dev)
     out = torch.full((L, B, HQ, D), float("nan"), dtype=torch.float32, device=cuda_dev)
     stream = torch.cuda.Stream()
-    for l in range(L):           # the benchmark's launch configuration
-        pool.decode_attention(l, q[l], tab_d, len_d, B, tab_d.shape[1], 1 / math.sqrt(D), out[l],
-                              stream)
+
+    def step(st, dst, overlap):
+        for l in range(L):
+            pool.decode_attention(l, q[l], tab_d, len_d, B, tab_d.shape[1], 1 / math.sqrt(D),
+                                  dst[l], st, overlap_previous=overlap and l > 0)
+
+    # the benchmark's launch configuration: one CUDA graph of the 48 per-layer
+    # calls, layers 1..47 overlapping the previous call
+    import bench
+    graph = bench.capture_graph(lambda st: step(st, out, True), stream)
+    assert graph is not None
+    out.fill_(float("nan"))
+    with torch.cuda.stream(stream):
+        graph.replay()
+    direct = torch.full_like(out, float("nan"))
+    step(stream, direct, False)                 # serialised calls, no graph
     torch.cuda.synchronize()
     assert pool.check_device() == 0
     assert torch.isfinite(out).all()
+    assert torch.equal(out, direct)
     rng = np.random.default_rng(7)
     full = [int(x) for x in rng.choice(B, size=2, replace=False)]
     layers_for = {b: (list(range(L)) if b in full else [int(rng.integers(0, L))]) for b in range(B)}
