@@ -134,8 +134,11 @@ class TraceDriver:
         sid = self.sids[i]
         t0 = self.tokens[i]
         if self.gpu:
-            k, v = self.kv_source(sid, t0, t0 + n)
-            kvtier.session_append(self.pool, sid, k, v, n, stream)
+            # produce the values on the stream that consumes them (side
+            # streams do not order against the default stream)
+            with self._torch.cuda.stream(stream):
+                k, v = self.kv_source(sid, t0, t0 + n)
+                kvtier.session_append(self.pool, sid, k, v, n, stream)
         else:
             kvtier.session_append(self.pool, sid, None, None, n, None)
         self.tokens[i] += n

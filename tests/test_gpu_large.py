@@ -101,6 +101,7 @@ def test_decode_full_size_bench_configuration(P, cuda_dev):
     len_d = torch.as_tensor(lens.astype(np.int32), device=cuda_dev)
     out = torch.full((L, B, HQ, D), float("nan"), dtype=torch.float32, device=cuda_dev)
     stream = torch.cuda.Stream()
+    torch.cuda.synchronize()     # the fill ran on the default stream
 
     def step(st, dst, overlap):
         for l in range(L):
@@ -140,6 +141,7 @@ def test_resume_burst_full_size(P, cuda_dev):
     for s in sids:
         synth.fill_image_torch(pool.image(s), seed, s, L, HKV, D, T)
     st = torch.cuda.Stream()
+    torch.cuda.synchronize()     # the fills ran on the default stream
     for s in sids:
         pool.session_resume(s, st)
     torch.cuda.synchronize()
@@ -168,6 +170,7 @@ def test_resume_burst_full_size(P, cuda_dev):
         pool.session_destroy(s)
     k, v = synth.kv_logical_torch(seed, 0, range(L), HKV, D, 0, T, cuda_dev)
     kk, vv = k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+    torch.cuda.synchronize()     # made on the default stream, appended on `st`
     fresh = [pool.session_create(T) for _ in range(n)]
     for s in fresh:
         pool.session_append(s, kk, vv, st)

@@ -150,6 +150,7 @@ def test_overlapped_calls_bit_identical(pkg):
     t = torch.as_tensor(tables, device=dev)
     s = torch.as_tensor(np.asarray(lens, dtype=np.int32), device=dev)
     st = torch.cuda.Stream()
+    torch.cuda.synchronize()     # inputs were made on the default stream
     outs = []
     for overlap in (False, True, True):
         out = torch.full((L, len(lens), 32, 128), float("nan"), dtype=torch.float32, device=dev)

@@ -44,6 +44,7 @@ def test_residency_random_sequence(cuda_dev):
     mb = -(-cap // bt)
     tables = torch.empty(4, mb, dtype=torch.int32, device=cuda_dev)
     slens = torch.empty(4, dtype=torch.int32, device=cuda_dev)
+    torch.cuda.synchronize()     # q was made on the default stream
     checked = 0
     for step in range(260):
         r = rnd.random()
@@ -51,7 +52,8 @@ def test_residency_random_sequence(cuda_dev):
             if rnd.random() < 0.5:
                 n0 = rnd.randint(20, 200)
                 sid = pool.session_create_paused(cap, n0)
-                synth.fill_image_torch(pool.image(sid), seed, sid, L, Hkv, D, n0)
+                with torch.cuda.stream(st):   # on the stream the pool's work uses
+                    synth.fill_image_torch(pool.image(sid), seed, sid, L, Hkv, D, n0)
                 o.create_paused(sid, cap, n0)
                 T[sid] = n0
             else:
@@ -79,9 +81,11 @@ def test_residency_random_sequence(cuda_dev):
                 o.append(sid, n)
             except NoHotBlocks:
                 continue
-            k, v = synth.kv_logical_torch(seed, sid, range(L), Hkv, D, T[sid], T[sid] + n, cuda_dev)
-            pool.session_append(sid, k.permute(0, 2, 1, 3).contiguous(),
-                                v.permute(0, 2, 1, 3).contiguous(), st)
+            with torch.cuda.stream(st):       # values made on the appending stream
+                k, v = synth.kv_logical_torch(seed, sid, range(L), Hkv, D, T[sid], T[sid] + n,
+                                              cuda_dev)
+                pool.session_append(sid, k.permute(0, 2, 1, 3).contiguous(),
+                                    v.permute(0, 2, 1, 3).contiguous(), st)
             T[sid] += n
         elif r < 0.7:
             o.pause(sid)
@@ -96,8 +100,8 @@ def test_residency_random_sequence(cuda_dev):
             except NoHotBlocks:
                 continue
             pool.batch_tables(batch, tables, mb, slens, st)
-            out = torch.empty(L, len(batch), Hq, D, dtype=torch.float32, device=cuda_dev)
             with torch.cuda.stream(st):
+                out = torch.empty(L, len(batch), Hq, D, dtype=torch.float32, device=cuda_dev)
                 pool.decode_attention(-1, q[:, :len(batch)].contiguous(), tables, slens, len(batch),
                                       mb, 1 / math.sqrt(D), out, st)
             torch.cuda.synchronize()

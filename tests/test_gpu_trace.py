@@ -52,6 +52,7 @@ def test_small_trace_parity(cuda_dev):
     tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=cuda_dev)
     seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=cuda_dev)
     dstream, mstream = torch.cuda.Stream(), torch.cuda.Stream()
+    torch.cuda.synchronize()     # inputs made on the default stream are complete
     checked = []
 
     def on_step(k, members):
@@ -88,4 +89,81 @@ def test_small_trace_parity(cuda_dev):
         img = pool.image(i)[:, :, :, :n].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
         k, v = synth.session_kv_np(cfg.seed, i, range(L), Hkv, D, n)
         assert np.array_equal(img[:, 0], k) and np.array_equal(img[:, 1], v)
+    pool.close()
+
+
+def test_full_trace_sampled_parity(cuda_dev):
+    """The benchmark's trace (48 sessions, N_a = 16, 2 000 steps, 48 layers),
+    with appended tokens taking their logical values so the oracle can
+    regenerate any session: at sampled steps two members of the batch are
+    checked on one layer each; at the end every image prefix is checked."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool, kvtier
+    from paper_2609_25782_gb300 import trace as tr
+
+    cfg = tr.TraceConfig(seed=0)
+    L, Hkv, Hq, D, bt = cfg.layers, cfg.num_kv_heads, cfg.num_q_heads, 128, cfg.block_tokens
+    trace = tr.generate(cfg)
+    plan = tr.plan(cfg, trace)
+    nb = plan["peak_blocks"] + 256
+    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=plan["cold_bytes"] + 4096,
+                max_sessions=cfg.sessions, max_batch=cfg.active_cap,
+                max_context=plan["max_context"], alloc_seed=cfg.seed)
+    for i, t in enumerate(trace):
+        sid = pool.session_create_paused(plan["caps"][i], t.t0)
+        synth.fill_image_torch(pool.image(sid), cfg.seed, sid, L, Hkv, D, t.t0)
+
+    def kv_source(sid, t0, t1):
+        k, v = synth.kv_logical_torch(cfg.seed, sid, range(L), Hkv, D, t0, t1, cuda_dev)
+        return k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+
+    q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(L), Hq, D, cuda_dev)
+    out = torch.empty(L, cfg.active_cap, Hq, D, dtype=torch.float32, device=cuda_dev)
+    max_blocks = -(-plan["max_context"] // bt)
+    tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=cuda_dev)
+    seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=cuda_dev)
+    torch.cuda.synchronize()     # inputs made on the default stream are complete
+    rng = np.random.default_rng(1)
+    sample_steps = {400, 1200, 1999}
+    checked = []
+
+    def on_step(k, members):
+        if k not in sample_steps:
+            return
+        torch.cuda.synchronize()
+        for r in rng.choice(len(members), size=2, replace=False):
+            m = members[int(r)]
+            l = int(rng.integers(0, L))
+            T = int(kvtier.session_info(pool.handle, m).tokens)
+            kk, vv = synth.session_kv_np(cfg.seed, m, [l], Hkv, D, T)
+            nblk = -(-T // bt)
+            host = np.full((nblk, 1, 2, Hkv, bt, D), synth.BF16_NAN, dtype=np.uint16)
+            for j in range(nblk):
+                n = min(bt, T - j * bt)
+                host[j, 0, 0, :, :n] = kk[0, :, j * bt:j * bt + n]
+                host[j, 0, 1, :, :n] = vv[0, :, j * bt:j * bt + n]
+            qh = q[l:l + 1, int(r):int(r) + 1].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+            ref = oracle.paged_decode(host, qh, np.arange(nblk, dtype=np.int32)[None], [T],
+                                      1 / math.sqrt(D), Hq)
+            got = out[l:l + 1, int(r):int(r) + 1].double().cpu().numpy()
+            err = np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref)))
+            assert err <= TOL, (k, m, l, err)
+            checked.append((k, m))
+
+    d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
+                       decode_stream=torch.cuda.Stream(priority=-1), mig_stream=torch.cuda.Stream(),
+                       tables=tables, seq_lens=seq_lens, max_blocks=max_blocks, on_step=on_step)
+    d.run()
+    torch.cuda.synchronize()
+    assert len(checked) == 6
+    assert d.counts == plan["counts"]
+    assert pool.check_device() == 0
+    # every image holds its session's logical KV for the packed prefix (sampled layers)
+    for i in range(cfg.sessions):
+        n = int(kvtier.session_info(pool.handle, i).cold_valid)
+        l = i % L
+        img = pool.image(i)[l, :, :, :n].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+        kk, vv = synth.session_kv_np(cfg.seed, i, [l], Hkv, D, n)
+        assert np.array_equal(img[0], kk[0]) and np.array_equal(img[1], vv[0])
     pool.close()
