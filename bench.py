@@ -550,10 +550,12 @@ def run_sweep(args):
         nb = max_tok // bt + 64
         Bmax = max(B for B, _ in pts)
         # workspace rows: the largest of layers x B x Hq x splits(T) over the points
-        need = max(L * B * HQ * -(-T // 2048) for B, T in pts)
+        def splits(t):    # the library's split bound for t tokens
+            return max(-(-t // 2048), min(16, -(-t // 1024)))
+        need = max(L * B * HQ * splits(T) for B, T in pts)
         ctx = max(SWEEP_T)
         pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,
-                    max_sessions=4, max_batch=-(-need // (HQ * -(-ctx // 2048))),
+                    max_sessions=4, max_batch=-(-need // (HQ * splits(ctx))),
                     max_context=ctx, device=dev.index)
         # values: one synthetic session laid over the whole pool (finite N(0,1))
         synth.fill_hot_pool_torch(pool.hot, args.seed, [0], [nb * bt], [np.arange(nb)], L, HKV, D,

@@ -187,8 +187,9 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  * The result depends only on the values and seq_lens: not on physical
  * placement, batch composition or timing (bit-identical across a
  * pause/resume round trip). The pool's decode workspace holds
- * max_batch x Hq x S(max_context) partial rows, S(t) = ceil(t / 2048) being
- * the number of 2 048-token splits of t tokens; a call needs
+ * max_batch x Hq x S(max_context) partial rows, S(t) being the split bound
+ * for t tokens (ceil(t / 1024) up to 16 splits, ceil(t / 2048) beyond 32K
+ * tokens); a call needs
  * layers x B x Hq x S(max_blocks x bt) rows, else KV_ERR_INVALID_ARG. Calls on
  * one pool share the workspace: issue them in order on one stream. */
 int decode_attention(kv_pool *pool, int32_t layer, const void *q,
@@ -291,8 +292,9 @@ int kv_pool_inject_cuda_failure(kv_pool *pool, int32_t n);
  * partials live in one file-scope device array of KV_NOALLOC_SCRATCH_BYTES
  * (48 MiB) that every GPU loading the library holds until the process exits.
  * A call needs layers x B x Hq x S x 520 bytes (+256), S the split count for
- * max_blocks * block_tokens tokens (ceil(t / 2048)); larger requests fail
- * with KV_ERR_INVALID_ARG before any work.
+ * max_blocks * block_tokens tokens (at most 16 up to 32K tokens,
+ * ceil(t / 2048) beyond); larger requests fail with KV_ERR_INVALID_ARG before
+ * any work.
  * It calls no cudaMalloc, cudaFree or allocating library routine.
  *
  * The first call on a device, with that device current, looks up the

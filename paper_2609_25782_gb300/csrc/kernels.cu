@@ -11,6 +11,8 @@
 //   migrate_kernel<false>  data path 2: resume-unpack, cold image -> blocks.
 //   migrate_kernel<true>   data path 4: pause-pack, blocks -> cold image,
 //                          tokens [t0, T) only (write-on-evict, Section 3).
+//   block_jobs_kernel<>    the same moves for explicit (slot, block, token
+//                          range) lists: residency-mode evictions and fetches.
 //   append_kernel          data path 3: fresh tokens into the tail blocks.
 //   table_write_kernel / gather_tables_kernel: block-table bookkeeping.
 //

@@ -22,11 +22,12 @@ constexpr int32_t kErrTimeout = 4;     // an mbarrier wait gave up
 // result never depends on batch composition or placement: split s covers
 // tiles [s*split_tiles, (s+1)*split_tiles) of the ceil(T/16) 16-token tiles.
 // split_tiles = clamp(ceil(tiles / 16), KVT_SPLIT_MIN_TILES, KVT_SPLIT_MAX_TILES).
-// The defaults fix it at 128 tiles (2 048 tokens): measured on GB300 against
-// 8..128-tile variants, it gives the highest bandwidth from 1K to 128K tokens
-// (fewer partials to merge, while 3 CTAs per SM keep the loads in flight).
+// The defaults, 64..128 tiles (1 024 tokens up to 16K-token sessions, growing
+// to 2 048 at 32K), come from GB300 measurements of 8..128-tile variants:
+// long splits leave few partials to merge, while 1 024-token splits keep
+// enough CTAs for the smaller batches of an agentic trace.
 #ifndef KVT_SPLIT_MIN_TILES
-#define KVT_SPLIT_MIN_TILES 128
+#define KVT_SPLIT_MIN_TILES 64
 #endif
 #ifndef KVT_SPLIT_MAX_TILES
 #define KVT_SPLIT_MAX_TILES 128

@@ -67,7 +67,7 @@ def host_hot(pool, seed, sess, lens, tables, k_scale=1.0):
 
 
 LENGTHS = [1, 2, 15, 16, 17, 31, 33, 63, 64, 65, 127, 128, 129, 255, 511, 512, 513, 1000,
-           1793, 2047, 2048, 2049, 4096, 4097, 6143, 8191, 8193]
+           1023, 1024, 1025, 1793, 2047, 2048, 2049, 4096, 4097, 6143, 8191, 8193, 17000]
 
 
 def test_decode_many_lengths_all_and_per_layer(pkg):
