@@ -205,6 +205,9 @@ int decode_attention(kv_pool *pool, int32_t layer, const void *q,
  * decode_attention call) does not write the hot arena, block_tables or
  * seq_lens. flags = 0 is decode_attention. */
 #define KV_DECODE_OVERLAP_PREVIOUS 1u
+/* KV_DECODE_OUT_BF16: `out` is bf16 [..][Hq][D] (the fp32 result rounded to
+ * nearest even), halving the output bytes for a caller that consumes bf16. */
+#define KV_DECODE_OUT_BF16 2u
 int decode_attention_ex(kv_pool *pool, int32_t layer, const void *q,
                         const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                         int32_t max_blocks, float scale, float *out, uint32_t flags,
@@ -261,11 +264,11 @@ int kv_pool_get_stats(kv_pool *pool, kv_pool_stats *out);
  * non-zero value makes the call return KV_ERR_DEVICE_CHECK. */
 int kv_pool_check_device(kv_pool *pool, int32_t *flags);
 
-/* Cap the migration kernels (resume-unpack, pause-pack, evictions) at about
- * max_ctas CTAs of 256 threads (rounded up to 8 per SM-sized unit), so that
- * migrations running beside decode take a smaller share of HBM bandwidth
- * (Section 3, data paths: eviction and resume overlap decode). 0 removes the
- * cap (the default: 8 CTAs per SM). Affects later calls only. */
+/* Cap the migration kernels (resume-unpack, pause-pack, evictions) at
+ * max_ctas CTAs of 256 threads, so that migrations running beside decode take
+ * a smaller share of HBM bandwidth (Section 3, data paths: eviction and resume
+ * overlap decode). 0 removes the cap (the default grid: 16 CTAs per SM).
+ * Affects later calls only. */
 int kv_pool_set_migration_limit(kv_pool *pool, int32_t max_ctas);
 
 /* Test hook: make the n-th following CUDA call of this pool fail (as a

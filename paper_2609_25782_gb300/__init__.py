@@ -105,10 +105,13 @@ class Pool:
 
     def decode_attention(self, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
                          scale: float, out, stream=None, overlap_previous: bool = False) -> None:
-        if overlap_previous:
+        """out: fp32, or bf16 (then the result is rounded to nearest even)."""
+        import torch
+        flags = (kvtier.KV_DECODE_OVERLAP_PREVIOUS if overlap_previous else 0) | \
+            (kvtier.KV_DECODE_OUT_BF16 if getattr(out, "dtype", None) == torch.bfloat16 else 0)
+        if flags:
             kvtier.decode_attention_ex(self.handle, layer, q, block_tables, seq_lens, B,
-                                       max_blocks, scale, out, kvtier.KV_DECODE_OVERLAP_PREVIOUS,
-                                       stream)
+                                       max_blocks, scale, out, flags, stream)
         else:
             kvtier.decode_attention(self.handle, layer, q, block_tables, seq_lens, B, max_blocks,
                                     scale, out, stream)

@@ -400,9 +400,20 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         }
         if (nsplit == 1) {
             const float inv = 1.f / lsum;
-            float4 *dst = reinterpret_cast<float4 *>(a.out + (row_base + h) * kHeadDim + d0);
-            dst[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
-            dst[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+            if (a.out_bf16) {
+                uint4 pk;
+                float r0, r1;
+                pk.x = pack_bf16(acc[0] * inv, acc[1] * inv, r0, r1);
+                pk.y = pack_bf16(acc[2] * inv, acc[3] * inv, r0, r1);
+                pk.z = pack_bf16(acc[4] * inv, acc[5] * inv, r0, r1);
+                pk.w = pack_bf16(acc[6] * inv, acc[7] * inv, r0, r1);
+                *reinterpret_cast<uint4 *>(reinterpret_cast<uint16_t *>(a.out) +
+                                           (row_base + h) * kHeadDim + d0) = pk;
+            } else {
+                float4 *dst = reinterpret_cast<float4 *>(a.out + (row_base + h) * kHeadDim + d0);
+                dst[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
+                dst[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+            }
         } else {
             const int64_t prow = (row_base + h) * a.max_splits + split;
             float4 *dst = reinterpret_cast<float4 *>(a.part_o + prow * kHeadDim + d0);
@@ -482,9 +493,37 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
             l += c * s_l[w];
         }
         const float inv = 1.f / l;
-        reinterpret_cast<float4 *>(a.out + row * kHeadDim)[lane] =
-            make_float4(r.x * inv, r.y * inv, r.z * inv, r.w * inv);
+        if (a.out_bf16) {
+            float r0, r1;
+            uint2 pk;
+            pk.x = pack_bf16(r.x * inv, r.y * inv, r0, r1);
+            pk.y = pack_bf16(r.z * inv, r.w * inv, r0, r1);
+            reinterpret_cast<uint2 *>(reinterpret_cast<uint16_t *>(a.out) + row * kHeadDim)[lane] = pk;
+        } else {
+            reinterpret_cast<float4 *>(a.out + row * kHeadDim)[lane] =
+                make_float4(r.x * inv, r.y * inv, r.z * inv, r.w * inv);
+        }
     }
+}
+
+// Migration copy shape, from GB300 measurements of 2..16 loads per lane and
+// 4..16 CTAs per SM: 4 loads per lane over a grid of 16 CTAs per SM moves an
+// 8 x 32K-token burst at 0.97-0.98 of the copy bandwidth (0.93 with 8 x 8).
+#ifndef KVT_MIG_UNROLL
+#define KVT_MIG_UNROLL 4          // 16-byte loads in flight per lane
+#endif
+#ifndef KVT_MIG_CTAS_PER_SM
+#define KVT_MIG_CTAS_PER_SM 16    // grid-stride CTAs of 256 threads per SM
+#endif
+
+__device__ __forceinline__ void st_out(uint4 *p, const uint4 &v) {
+#ifdef KVT_MIG_STREAM_STORE
+    asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+#else
+    *p = v;
+#endif
 }
 
 __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
@@ -497,7 +536,7 @@ __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
 
 // K3 / K4: one warp per (layer, K|V, kv-head, block) run of the token range.
 // Both sides of a run are contiguous rows of 256 B; a warp moves it with
-// 16-byte loads, eight in flight per lane. Items are ordered run-major so
+// 16-byte loads, KVT_MIG_UNROLL in flight per lane. Items are ordered run-major so
 // that consecutive warps walk the image sequentially.
 template <bool kPack>
 __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
@@ -525,17 +564,17 @@ __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
         const uint4 *src = reinterpret_cast<const uint4 *>(kPack ? hp : ip);
         uint4 *dst = reinterpret_cast<uint4 *>(kPack ? ip : hp);
         const int units = (t_hi - t_lo) * (kRowBytes / 16);
-        for (int u0 = 0; u0 < units; u0 += 32 * 8) {
-            uint4 v[8];
+        for (int u0 = 0; u0 < units; u0 += 32 * KVT_MIG_UNROLL) {
+            uint4 v[KVT_MIG_UNROLL];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
                 const int u = u0 + k * 32 + lane;
                 if (u < units) v[k] = ld_stream(src + u);
             }
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
                 const int u = u0 + k * 32 + lane;
-                if (u < units) dst[u] = v[k];
+                if (u < units) st_out(dst + u, v[k]);
             }
         }
     }
@@ -564,17 +603,17 @@ __global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__
         const uint4 *src = reinterpret_cast<const uint4 *>(kPack ? hp : ip);
         uint4 *dst = reinterpret_cast<uint4 *>(kPack ? ip : hp);
         const int units = (b.t1 - b.t0) * (kRowBytes / 16);
-        for (int u0 = 0; u0 < units; u0 += 32 * 8) {
-            uint4 v[8];
+        for (int u0 = 0; u0 < units; u0 += 32 * KVT_MIG_UNROLL) {
+            uint4 v[KVT_MIG_UNROLL];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
                 const int u = u0 + k * 32 + lane;
                 if (u < units) v[k] = ld_stream(src + u);
             }
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
                 const int u = u0 + k * 32 + lane;
-                if (u < units) dst[u] = v[k];
+                if (u < units) st_out(dst + u, v[k]);
             }
         }
     }
@@ -689,38 +728,44 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStrea
     return cudaLaunchKernelEx(&c2, decode_combine_kernel, a);
 }
 
-static unsigned mig_grid(int64_t items, int num_sms) {
+// One warp per item, 8 per CTA; at most KVT_MIG_CTAS_PER_SM per SM, or
+// max_ctas when the caller caps migrations (max_ctas > 0).
+static unsigned mig_grid(int64_t items, int num_sms, int max_ctas) {
     int64_t blocks = (items + 7) / 8;
-    const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+    int64_t cap = static_cast<int64_t>(num_sms) * KVT_MIG_CTAS_PER_SM;
+    if (max_ctas > 0 && max_ctas < cap) cap = max_ctas;
     if (blocks > cap) blocks = cap;
     return static_cast<unsigned>(blocks < 1 ? 1 : blocks);
 }
 
-cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st) {
+cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st) {
     if (a.t_end <= a.t_begin) return cudaSuccess;
     const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
-    migrate_kernel<false><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms), 256, 0, st>>>(a);
+    migrate_kernel<false><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
-cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st) {
+cudaError_t launch_pack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st) {
     if (a.t_end <= a.t_begin) return cudaSuccess;
     const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
-    migrate_kernel<true><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms), 256, 0, st>>>(a);
+    migrate_kernel<true><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st) {
     const int64_t warps = static_cast<int64_t>(a.s.L) * a.n;
     int64_t blocks = (warps + 7) / 8;
-    if (blocks > static_cast<int64_t>(num_sms) * 8) blocks = static_cast<int64_t>(num_sms) * 8;
+    const int64_t cap = static_cast<int64_t>(num_sms) * KVT_MIG_CTAS_PER_SM;
+    if (blocks > cap) blocks = cap;
     append_kernel<<<static_cast<unsigned>(blocks < 1 ? 1 : blocks), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
-cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, cudaStream_t st) {
+cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, int max_ctas,
+                              cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    const unsigned grid = mig_grid(static_cast<int64_t>(a.n) * a.s.L * 2 * a.s.Hkv, num_sms);
+    const unsigned grid =
+        mig_grid(static_cast<int64_t>(a.n) * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas);
     if (pack)
         block_jobs_kernel<true><<<grid, 256, 0, st>>>(a);
     else

@@ -62,12 +62,13 @@ struct DecodeArgs {
     const uint16_t *q;        // [nl][B][Hq][D] bf16
     const int32_t *tables;    // [B][max_blocks]
     const int32_t *seq_lens;  // [B]
-    float *out;               // [nl][B][Hq][D]
+    float *out;               // [nl][B][Hq][D], fp32 or (out_bf16) bf16
     float *part_o;            // [nl*B][Hq][max_splits][D]
     float *part_ml;           // [nl*B][Hq][max_splits][2]
     int32_t *err;
     int32_t B, max_blocks, layer0, nlayers, max_splits;
     float scale_log2;         // scale * log2(e)
+    int32_t out_bf16;         // 1: out holds bf16 (round to nearest even)
     Shape s;
 };
 
@@ -136,10 +137,12 @@ cudaError_t prepare_kernels();  // per-device function attributes
 // previous kernel on the stream (see decode_attention_ex).
 cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st,
                           bool overlap_previous);
-cudaError_t launch_unpack(const MigArgs &a, int num_sms, cudaStream_t st);
-cudaError_t launch_pack(const MigArgs &a, int num_sms, cudaStream_t st);
+// max_ctas > 0 caps the migration grids (kv_pool_set_migration_limit).
+cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);
+cudaError_t launch_pack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);
-cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, cudaStream_t st);
+cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, int max_ctas,
+                              cudaStream_t st);
 cudaError_t launch_table_write(const TableWriteArgs &a, cudaStream_t st);
 cudaError_t launch_gather(const GatherArgs &a, cudaStream_t st);
 

@@ -100,13 +100,6 @@ struct kv_pool {
     int mig_ctas = 0;                    // cap on migration-kernel CTAs, 0 = none
     kvt::Shape shape{};
 
-    // SM budget handed to the migration kernels (8 CTAs per unit).
-    int mig_units() const {
-        if (mig_ctas <= 0) return num_sms;
-        const int u = (mig_ctas + 7) / 8;
-        return u < 1 ? 1 : u;
-    }
-
     std::vector<int32_t> free_list;      // top = back
     std::vector<int16_t> block_fence;    // fence slot of the pack that freed it, or -1
     std::vector<uint64_t> block_fence_gen;
@@ -324,7 +317,7 @@ struct kv_pool {
             a.pad = 0;
             std::copy(jobs.begin() + i, jobs.begin() + i + a.n, a.job);
             int rc = cuda(pack ? "pack launch" : "unpack launch",
-                          [&] { return kvt::launch_block_jobs(a, pack, mig_units(), st); });
+                          [&] { return kvt::launch_block_jobs(a, pack, num_sms, mig_ctas, st); });
             if (rc) return rc;
         }
         return KV_OK;
@@ -777,7 +770,7 @@ int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *bl
 int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
                         const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
                         float *out, uint32_t flags, kv_stream_t stream_) {
-    if (flags & ~static_cast<uint32_t>(KV_DECODE_OVERLAP_PREVIOUS))
+    if (flags & ~static_cast<uint32_t>(KV_DECODE_OVERLAP_PREVIOUS | KV_DECODE_OUT_BF16))
         return fail(KV_ERR_INVALID_ARG, "unknown decode flag");
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
@@ -810,6 +803,7 @@ int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t 
     a.nlayers = nl;
     a.max_splits = splits;
     a.scale_log2 = scale * 1.4426950408889634f;
+    a.out_bf16 = (flags & KV_DECODE_OUT_BF16) ? 1 : 0;
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     const bool overlap = (flags & KV_DECODE_OVERLAP_PREVIOUS) != 0;
@@ -847,7 +841,7 @@ int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
         kvt::MigArgs m = p->mig_args(sid, *s);
         m.t_begin = static_cast<int32_t>(t0);
         m.t_end = static_cast<int32_t>(t1);
-        rc = p->cuda("pack launch", [&] { return kvt::launch_pack(m, p->mig_units(), st); });
+        rc = p->cuda("pack launch", [&] { return kvt::launch_pack(m, p->num_sms, p->mig_ctas, st); });
     }
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(p->fences[f].ev, st); });
     if (rc) return rc;
@@ -894,7 +888,7 @@ int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
         kvt::MigArgs m = p->mig_args(sid, *s);
         m.t_begin = 0;
         m.t_end = static_cast<int32_t>(s->T);
-        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->mig_units(), st); });
+        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->num_sms, p->mig_ctas, st); });
     }
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
     if (rc) return rc;

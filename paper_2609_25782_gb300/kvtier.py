@@ -41,6 +41,7 @@ EXPORTS = [
 ]
 
 KV_DECODE_OVERLAP_PREVIOUS = 1
+KV_DECODE_OUT_BF16 = 2
 
 KV_NOALLOC_SCRATCH_BYTES = 48 << 20
 

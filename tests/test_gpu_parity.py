@@ -169,6 +169,27 @@ def test_overlapped_calls_bit_identical(pkg):
     assert pool.check_device() == 0
 
 
+def test_bf16_output_is_rounded_fp32(pkg):
+    """KV_DECODE_OUT_BF16: each output is the fp32 result rounded to nearest
+    even, both from one-split sessions (split kernel) and merged ones."""
+    lens = [5, 700, 2047, 5000, 13000]
+    pool, sess, tables, q = direct_case(pkg, lens, L=2, seed=14)
+    dev = torch.device("cuda:0")
+    t = torch.as_tensor(tables, device=dev)
+    s = torch.as_tensor(np.asarray(lens, dtype=np.int32), device=dev)
+    o32 = torch.empty(2, len(lens), 32, 128, dtype=torch.float32, device=dev)
+    o16 = torch.empty(2, len(lens), 32, 128, dtype=torch.bfloat16, device=dev)
+    pool.decode_attention(-1, q, t, s, len(lens), t.shape[1], 1 / math.sqrt(128), o32)
+    pool.decode_attention(-1, q, t, s, len(lens), t.shape[1], 1 / math.sqrt(128), o16)
+    torch.cuda.synchronize()
+    assert torch.equal(o16.view(torch.int16), o32.to(torch.bfloat16).view(torch.int16))
+    ref = oracle.paged_decode(host_hot(pool, 14, sess, lens, tables),
+                              q.cpu().view(torch.int16).numpy().view(np.uint16), tables, lens,
+                              1 / math.sqrt(128), 32)
+    assert scaled_err(o16.double().cpu().numpy(), ref) <= TOL
+    assert pool.check_device() == 0
+
+
 def test_nan_tail_slots_do_not_leak(pkg):
     lens = [17, 100, 529]
     pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=6)
