@@ -423,7 +423,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     from paper_2609_25782_gb300 import trace as tr
     dev = torch.device("cuda", torch.cuda.current_device())
     cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps,
-                         admit_lead=args.trace_admit_lead)
+                         admit_lead=args.trace_admit_lead,
+                         fused_append=not args.trace_unfused_append)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -453,6 +454,11 @@ def run_trace(args, rank, lru_factor: float = 0.0):
         shape = (cfg.layers, n, cfg.num_kv_heads, D)
         return flat_k[: n * per_tok].view(shape), flat_v[: n * per_tok].view(shape)
 
+    def kv_step_source(sids, positions):     # the step tokens of a batch, [L][B][Hkv][D]
+        shape = (cfg.layers, len(sids), cfg.num_kv_heads, D)
+        n = len(sids) * per_tok
+        return flat_k[:n].view(shape), flat_v[:n].view(shape)
+
     q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(cfg.layers), HQ, D, dev)
     out = torch.empty(cfg.layers, cfg.active_cap, HQ, D, dtype=torch.float32, device=dev)
     max_blocks = -(-plan["max_context"] // cfg.block_tokens)
@@ -463,7 +469,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     torch.cuda.synchronize()
     d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
                        decode_stream=dstream, mig_stream=mstream, tables=tables,
-                       seq_lens=seq_lens, max_blocks=max_blocks)
+                       seq_lens=seq_lens, max_blocks=max_blocks, kv_step_source=kv_step_source)
     t0 = time.perf_counter()
     with torch.cuda.stream(dstream):
         d.run()
@@ -508,6 +514,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     return {
         **extra,
         "admit_lead": cfg.admit_lead, "mig_ctas": args.trace_mig_ctas,
+        "step_append": "fused into the decode kernel" if cfg.fused_append else "separate kernel",
         "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
         "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
         "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2),
@@ -732,6 +739,10 @@ def main():
                     help="steps between a session's resume and its first decode step")
     ap.add_argument("--trace-mig-ctas", type=int, default=0,
                     help="cap on migration-kernel CTAs during the trace (0: none)")
+    ap.add_argument("--only-trace", action="store_true",
+                    help="run only the agentic trace (simple and residency modes)")
+    ap.add_argument("--trace-unfused-append", action="store_true",
+                    help="trace: write each step's token with its own kernel before the decode")
     ap.add_argument("--no-trace", action="store_true")
     ap.add_argument("--graph", action=argparse.BooleanOptionalAction, default=True,
                     help="replay the per-layer calls of a step from one CUDA graph")
@@ -768,6 +779,12 @@ def main():
         sec = run_migration(args, rank)
         if rank == 0:
             print(json.dumps({"secondary": sec}))
+        return 0
+    if args.only_trace:
+        tr_res = {"trace": run_trace(args, rank),
+                  "trace_lru": run_trace(args, rank, lru_factor=1.5)}
+        if rank == 0:
+            print(json.dumps(tr_res))
         return 0
     res = run_decode(args, ws, rank)
     total_ms = res["total_ms"]

@@ -7,6 +7,8 @@
  *   path 1  decode attention over the HBM-resident hot set ... decode_attention
  *   path 2  resume: cold image -> hot blocks ................ session_resume
  *   path 3  fresh KV written into hot blocks ................ session_append
+ *           (or kv_pool_batch_reserve + decode_append_attention: one
+ *           token per session and step, written by the decode kernel)
  *   path 4  eviction: hot blocks -> cold image .............. session_pause
  * The cold tier (high bandwidth flash in the paper) is a second device
  * allocation; its bandwidth, energy and endurance are not modelled.
@@ -200,10 +202,12 @@ int decode_attention(kv_pool *pool, int32_t layer, const void *q,
  * call's split kernel start while the kernel just before it on the stream is
  * still running (programmatic dependent launch): it reads block ids and
  * prefetches K/V tiles at once, and waits for that kernel to finish before
- * it reads q or writes out or the workspace. The caller promises that the
- * kernel just before it on the stream (typically the previous layer's
- * decode_attention call) does not write the hot arena, block_tables or
- * seq_lens. flags = 0 is decode_attention. */
+ * it reads q (or k_new, v_new) or writes out, the workspace or the pool. The
+ * caller promises that the kernel just before it on the stream (typically
+ * the previous layer's decode call) writes neither block_tables, seq_lens
+ * nor any hot-arena row of the layers this call reads; a
+ * decode_append_attention call for another layer writes only its own
+ * layer's rows and qualifies. flags = 0 is decode_attention. */
 #define KV_DECODE_OVERLAP_PREVIOUS 1u
 /* KV_DECODE_OUT_BF16: `out` is bf16 [..][Hq][D] (the fp32 result rounded to
  * nearest even), halving the output bytes for a caller that consumes bf16. */
@@ -212,6 +216,23 @@ int decode_attention_ex(kv_pool *pool, int32_t layer, const void *q,
                         const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                         int32_t max_blocks, float scale, float *out, uint32_t flags,
                         kv_stream_t stream);
+
+/* Data paths 3 and 1 fused (Section 3: the step's fresh KV is written into
+ * HBM and decode reads it): decode_attention_ex where the newest token of
+ * every batch row, position seq_lens[b] - 1, arrives with the call.
+ *   k_new, v_new  device bf16 [B][Hkv][D] (or [L][B][Hkv][D] for layer =
+ *                 -1), 16-byte aligned: that token's K and V
+ * The kernel stores them into the token's pool slot, which
+ * kv_pool_batch_reserve allocated (block_tables and seq_lens are its
+ * outputs), and attends over tokens 0 .. seq_lens[b] - 1 including it.
+ * Result and pool contents are bit-identical to session_append of the token
+ * followed by decode_attention_ex. Issue it for every layer (or once with
+ * layer = -1) before any call that may pack the sessions' blocks. Errors as
+ * decode_attention_ex; null or misaligned k_new/v_new -> KV_ERR_INVALID_ARG. */
+int decode_append_attention(kv_pool *pool, int32_t layer, const void *q, const void *k_new,
+                            const void *v_new, const int32_t *block_tables,
+                            const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
+                            float *out, uint32_t flags, kv_stream_t stream);
 
 /* Data path 4 with write-on-evict (Section 3, "Memory hierarchy and write
  * policy"): copy tokens [cold_valid, T) of an ACTIVE session into its
@@ -248,6 +269,25 @@ int session_block_table(kv_pool *pool, int32_t sid, int32_t *host_row, int32_t c
  * of B ids. */
 int kv_pool_batch_tables(kv_pool *pool, const int32_t *sids, int32_t B, int32_t *block_tables,
                          int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream);
+
+/* Data path 3 for one decode step of a batch, the values written by the
+ * decode kernel (decode_append_attention): each of the B distinct ACTIVE
+ * sessions in sids gets position T (a block is popped when its tail block
+ * is full) and T += 1; then block_tables and seq_lens are built as by
+ * kv_pool_batch_tables, so seq_lens[b] counts the new token. In residency
+ * mode the members' evicted blocks are fetched back first and victims come
+ * only from sessions outside the batch; all members are stamped with one
+ * recency time. Free-list pops go in batch order: a member's missing blocks
+ * in ascending order, then its new block. The stream first waits for the
+ * members' last resumes and for packs of popped blocks. Until the decode
+ * has written the new tokens their slots hold stale data, so no call that
+ * may pack these sessions (a pause, an eviction by a later allocation) may
+ * come before it. Errors: a session twice, paused or at capacity, or
+ * max_blocks too short -> KV_ERR_INVALID_ARG / KV_ERR_BAD_STATE;
+ * KV_ERR_NO_HOT_BLOCKS. All or nothing. Host-logic-only pools do the
+ * bookkeeping and ignore the outputs. */
+int kv_pool_batch_reserve(kv_pool *pool, const int32_t *sids, int32_t B, int32_t *block_tables,
+                          int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream);
 
 /* Re-run the Fisher-Yates shuffle over the current free list with a new
  * seed (scrambles where the next allocations land). */

@@ -164,6 +164,35 @@ class ResidencyOracle:
         for sid in sids:
             self.s[sid].time = t
 
+    def batch_reserve(self, sids: list):
+        """One decode step's fresh token for each session of the batch (its
+        values are written by the decode itself): evicted blocks come back,
+        a session whose tail block is full gets a new one, and every member
+        grows by one token. Victims are outside the batch; pops go member by
+        member, missing blocks first."""
+        assert len(set(sids)) == len(sids)
+        plan = []
+        for sid in sids:
+            s = self.s[sid]
+            assert s.state == "active" and s.T + 1 <= s.cap
+            missing = [j for j, slot in enumerate(s.slots) if slot < 0]
+            plan.append((sid, missing, 1 if s.T % self.bt == 0 else 0))
+        total = sum(len(m) + g for _, m, g in plan)
+        self._check_room(total, set(sids))
+        self._evict(total, set(sids))
+        for sid, missing, grow in plan:
+            s = self.s[sid]
+            if missing:
+                self._fetch(sid, missing)
+            if grow:
+                s.slots.append(int(self.fl.pop(1)[0]))
+                s.img.append(0)
+            s.T += 1
+            self.stats["bytes_appended"] += self.tb
+        t = self._tick()
+        for sid in sids:
+            self.s[sid].time = t
+
     def destroy(self, sid: int):
         s = self.s.pop(sid)
         self.fl.push([slot for slot in s.slots if slot >= 0])

@@ -103,6 +103,12 @@ class Pool:
         kvtier.kv_pool_batch_tables(self.handle, list(sids), block_tables, max_blocks, seq_lens,
                                     stream)
 
+    def batch_reserve(self, sids, block_tables, max_blocks: int, seq_lens, stream=None) -> None:
+        """One new position per session (filled by decode_append_attention),
+        then the batch's tables and lengths as batch_tables builds them."""
+        kvtier.kv_pool_batch_reserve(self.handle, list(sids), block_tables, max_blocks, seq_lens,
+                                     stream)
+
     def decode_attention(self, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
                          scale: float, out, stream=None, overlap_previous: bool = False) -> None:
         """out: fp32, or bf16 (then the result is rounded to nearest even)."""
@@ -115,6 +121,17 @@ class Pool:
         else:
             kvtier.decode_attention(self.handle, layer, q, block_tables, seq_lens, B, max_blocks,
                                     scale, out, stream)
+
+    def decode_append_attention(self, layer: int, q, k_new, v_new, block_tables, seq_lens, B: int,
+                                max_blocks: int, scale: float, out, stream=None,
+                                overlap_previous: bool = False) -> None:
+        """k_new, v_new: device bf16 [B][Hkv][D] (leading [L] for layer -1), the
+        token at seq_lens[b] - 1 of each row, written to the pool and attended to."""
+        import torch
+        flags = (kvtier.KV_DECODE_OVERLAP_PREVIOUS if overlap_previous else 0) | \
+            (kvtier.KV_DECODE_OUT_BF16 if getattr(out, "dtype", None) == torch.bfloat16 else 0)
+        kvtier.decode_append_attention(self.handle, layer, q, k_new, v_new, block_tables, seq_lens,
+                                       B, max_blocks, scale, out, flags, stream)
 
     def shuffle_free(self, seed: int) -> None:
         kvtier.kv_pool_shuffle_free(self.handle, seed)

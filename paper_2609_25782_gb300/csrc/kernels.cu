@@ -265,6 +265,31 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         const int ti = tile0 + warp + k * kDecodeWarps;
         const int tok_base = ti * kTileTokens;
 
+        if (a.k_new != nullptr && tok_base + kTileTokens >= T) {
+            // Fused append: token T-1 arrives with this call. Its K and V rows
+            // replace whatever the copy brought for that slot and are stored
+            // to the reserved pool slot. Lanes 0-15 move K, 16-31 V, 16 B each.
+            const int r = T - 1 - tok_base;
+            const int u = lane & 15;
+            const int isv = lane >> 4;
+            const uint4 val = *reinterpret_cast<const uint4 *>(
+                (isv ? a.v_new : a.k_new) +
+                ((static_cast<int64_t>(li) * a.B + b) * sh.Hkv + g) * kHeadDim + u * 8);
+            *reinterpret_cast<uint4 *>(ring + (k % kStages) * kTileBytes + isv * 2 * kHalfBytes +
+                                       (u >> 3) * kHalfBytes + swz(r, u & 7)) = val;
+            const int j = (T - 1) / sh.bt;
+            const int blk = trow[j];
+            if (blk >= 0 && blk < sh.num_blocks) {   // a bad id was flagged by the copy
+                const int64_t row =
+                    ((static_cast<int64_t>(blk) * sh.L + l) * 2 * sh.Hkv + g) * sh.bt +
+                    (T - 1 - j * sh.bt) + isv * chunk_rows;
+                *reinterpret_cast<uint4 *>(a.hot + row * kHeadDim + u * 8) = val;
+            }
+            // The slot is refilled by the async proxy later.
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+        }
+
         // S^T = K . Q^T, two accumulators to shorten the mma chain.
         float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll

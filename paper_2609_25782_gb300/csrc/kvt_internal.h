@@ -69,6 +69,11 @@ struct DecodeArgs {
     int32_t B, max_blocks, layer0, nlayers, max_splits;
     float scale_log2;         // scale * log2(e)
     int32_t out_bf16;         // 1: out holds bf16 (round to nearest even)
+    // Fused append (data path 3): when k_new is set, token seq_lens[b]-1 of
+    // each row arrives with the call, bf16 [nl][B][Hkv][D] each, and is
+    // written into its reserved pool slot as well as attended to.
+    const uint16_t *k_new, *v_new;
+    uint16_t *hot;            // pool base, written only when k_new is set
     Shape s;
 };
 

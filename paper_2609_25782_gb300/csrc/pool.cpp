@@ -767,9 +767,10 @@ int decode_attention(kv_pool *p, int32_t layer, const void *q, const int32_t *bl
                                stream_);
 }
 
-int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
-                        const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
-                        float *out, uint32_t flags, kv_stream_t stream_) {
+static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_new,
+                       const void *v_new, const int32_t *block_tables, const int32_t *seq_lens,
+                       int32_t B, int32_t max_blocks, float scale, float *out, uint32_t flags,
+                       kv_stream_t stream_) {
     if (flags & ~static_cast<uint32_t>(KV_DECODE_OVERLAP_PREVIOUS | KV_DECODE_OUT_BF16))
         return fail(KV_ERR_INVALID_ARG, "unknown decode flag");
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
@@ -804,6 +805,9 @@ int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t 
     a.max_splits = splits;
     a.scale_log2 = scale * 1.4426950408889634f;
     a.out_bf16 = (flags & KV_DECODE_OUT_BF16) ? 1 : 0;
+    a.k_new = static_cast<const uint16_t *>(k_new);
+    a.v_new = static_cast<const uint16_t *>(v_new);
+    a.hot = static_cast<uint16_t *>(p->cfg.hot_base);
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     const bool overlap = (flags & KV_DECODE_OVERLAP_PREVIOUS) != 0;
@@ -811,6 +815,24 @@ int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t 
     if (rc) return rc;
     p->stats.decodes += 1;
     return KV_OK;
+}
+
+int decode_attention_ex(kv_pool *p, int32_t layer, const void *q, const int32_t *block_tables,
+                        const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
+                        float *out, uint32_t flags, kv_stream_t stream) {
+    return decode_impl(p, layer, q, nullptr, nullptr, block_tables, seq_lens, B, max_blocks,
+                       scale, out, flags, stream);
+}
+
+int decode_append_attention(kv_pool *p, int32_t layer, const void *q, const void *k_new,
+                            const void *v_new, const int32_t *block_tables,
+                            const int32_t *seq_lens, int32_t B, int32_t max_blocks, float scale,
+                            float *out, uint32_t flags, kv_stream_t stream) {
+    if (!k_new || !v_new) return fail(KV_ERR_INVALID_ARG, "null k_new or v_new");
+    if ((reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new)) & 15)
+        return fail(KV_ERR_INVALID_ARG, "k_new and v_new must be 16-byte aligned");
+    return decode_impl(p, layer, q, k_new, v_new, block_tables, seq_lens, B, max_blocks, scale,
+                       out, flags, stream);
 }
 
 int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
@@ -936,6 +958,31 @@ int session_block_table(kv_pool *p, int32_t sid, int32_t *host_row, int32_t cap,
     return KV_OK;
 }
 
+// Device inputs of a decode batch from the pool's tables: row b of
+// block_tables (entries past the session's length set to -1) and seq_lens.
+static int gather_batch(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
+                        int32_t max_blocks, int32_t *seq_lens, cudaStream_t st) {
+    for (int32_t r0 = 0; r0 < B; r0 += kvt::kGatherMax) {
+        kvt::GatherArgs a;
+        a.arena = p->d_tables;
+        a.stride = p->table_stride;
+        a.tables = block_tables;
+        a.seq_lens = seq_lens;
+        a.max_blocks = max_blocks;
+        a.row0 = r0;
+        a.count = std::min(B - r0, kvt::kGatherMax);
+        for (int32_t i = 0; i < a.count; ++i) {
+            const Session &s = p->sessions[sids[r0 + i]];
+            a.sids[i] = sids[r0 + i];
+            a.lens[i] = static_cast<int32_t>(s.T);
+            a.nblk[i] = static_cast<int32_t>(s.blocks.size());
+        }
+        int rc = p->cuda("gather launch", [&] { return kvt::launch_gather(a, st); });
+        if (rc) return rc;
+    }
+    return KV_OK;
+}
+
 int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
                          int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream_) {
     if (!p || !sids || B < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
@@ -957,25 +1004,109 @@ int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *bl
         int rc = lru_fetch_batch(p, sids, B, st);
         if (rc || p->host_only) return rc;   // host-logic pools: bookkeeping only
     }
-    for (int32_t r0 = 0; r0 < B; r0 += kvt::kGatherMax) {
-        kvt::GatherArgs a;
-        a.arena = p->d_tables;
-        a.stride = p->table_stride;
-        a.tables = block_tables;
-        a.seq_lens = seq_lens;
-        a.max_blocks = max_blocks;
-        a.row0 = r0;
-        a.count = std::min(B - r0, kvt::kGatherMax);
-        for (int32_t i = 0; i < a.count; ++i) {
-            const Session &s = p->sessions[sids[r0 + i]];
-            a.sids[i] = sids[r0 + i];
-            a.lens[i] = static_cast<int32_t>(s.T);
-            a.nblk[i] = static_cast<int32_t>(s.blocks.size());
-        }
-        int rc = p->cuda("gather launch", [&] { return kvt::launch_gather(a, st); });
-        if (rc) return rc;
+    return gather_batch(p, sids, B, block_tables, max_blocks, seq_lens, st);
+}
+
+// Path 3 for one decode step: every member gets position T (a fresh block
+// when its tail block is full) and, in residency mode, its evicted blocks
+// back; victims come only from sessions outside the batch. The values
+// arrive with decode_append_attention. Free-list pops go in batch order:
+// a member's missing blocks (ascending), then its fresh block.
+int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
+                          int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream_) {
+    if (!p || !sids || B < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
+    if (!p->host_only && (!block_tables || !seq_lens)) return fail(KV_ERR_INVALID_ARG, "null output");
+    if (max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "max_blocks must be >= 1");
+    const int bt = p->cfg.block_tokens;
+    const std::vector<int32_t> members(sids, sids + B);
+    for (int32_t i = 0; i < B; ++i) {
+        Session *s = p->session(sids[i]);
+        if (!s) return fail(KV_ERR_INVALID_ARG, "no such session in batch");
+        if (std::find(members.begin(), members.begin() + i, sids[i]) != members.begin() + i)
+            return fail(KV_ERR_INVALID_ARG, "a session appears twice in the batch");
+        if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "paused session in batch");
+        if (s->T + 1 > s->cap) return fail(KV_ERR_INVALID_ARG, "append past the session capacity");
+        if ((s->T + bt) / bt > max_blocks)
+            return fail(KV_ERR_INVALID_ARG, "max_blocks shorter than a session's table");
     }
-    return KV_OK;
+    std::vector<std::vector<int32_t>> miss(B);
+    std::vector<char> grow(B);
+    int64_t need = 0;
+    for (int32_t i = 0; i < B; ++i) {
+        const Session &s = p->sessions[sids[i]];
+        if (p->lru)
+            for (size_t j = 0; j < s.blocks.size(); ++j)
+                if (s.blocks[j] < 0) miss[i].push_back(static_cast<int32_t>(j));
+        grow[i] = (s.T % bt) == 0;
+        need += static_cast<int64_t>(miss[i].size()) + grow[i];
+    }
+    std::vector<Victim> vic;
+    if (p->lru ? !p->plan_evict(need, members, vic)
+               : need > static_cast<int64_t>(p->free_list.size()))
+        return fail(KV_ERR_NO_HOT_BLOCKS, "the batch's blocks and new positions do not fit in the hot pool");
+    const std::vector<int32_t> got = p->peek_alloc(need, vic);
+    std::vector<std::vector<int32_t>> rows(B);
+    std::vector<int64_t> first(B);   // first changed table entry per member
+    std::vector<kvt::BlockJob> jobs;
+    std::vector<int32_t> fresh;      // popped slots that are not eviction victims
+    int64_t k = 0, fetched = 0;
+    for (int32_t i = 0; i < B; ++i) {
+        const Session &s = p->sessions[sids[i]];
+        rows[i] = s.blocks;
+        first[i] = static_cast<int64_t>(s.blocks.size());
+        for (int32_t j : miss[i]) {
+            rows[i][j] = got[k];
+            jobs.push_back(p->job_for(sids[i], j, got[k], 0, p->tokens_in_block(s, j)));
+            fetched += p->tokens_in_block(s, j);
+            first[i] = std::min<int64_t>(first[i], j);
+            ++k;
+        }
+        if (grow[i]) rows[i].push_back(got[k++]);
+    }
+    // Slots that come off the free list (not from this call's victims) may
+    // have been freed by a pause whose pack is still running.
+    for (int64_t i = 0; i < need && i < static_cast<int64_t>(p->free_list.size()); ++i)
+        fresh.push_back(p->free_list[p->free_list.size() - 1 - i]);
+
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
+    int rc = KV_OK;
+    for (int32_t i = 0; !rc && i < B; ++i) {
+        const Session &s = p->sessions[sids[i]];
+        if (s.ready_recorded) rc = wait_event(p, st, s.ready);
+    }
+    if (!rc && !fresh.empty()) rc = p->wait_fences(fresh.data(), fresh.size(), st);
+    if (!rc) rc = p->evict_device(vic, st);
+    if (!rc) rc = p->run_jobs(jobs, false, st);
+    for (int32_t i = 0; !rc && i < B; ++i) {
+        const int64_t n = static_cast<int64_t>(rows[i].size()) - first[i];
+        if (n > 0) rc = p->write_table(sids[i], rows[i].data() + first[i], first[i], n, st);
+    }
+    if (rc) return rc;   // host state untouched
+
+    p->evict_commit(vic);
+    p->free_list.resize(p->free_list.size() - need);
+    p->clear_fences(fresh.data(), fresh.size());
+    const uint64_t stamp = ++p->clock;
+    for (int32_t i = 0; i < B; ++i) {
+        Session &s = p->sessions[sids[i]];
+        if (p->lru) p->lru_out(sids[i]);
+        s.blocks = rows[i];
+        if (grow[i] && p->lru) s.img_tok.push_back(0);
+        s.T += 1;
+        if (p->lru) {
+            s.hot_count += static_cast<int64_t>(miss[i].size()) + grow[i];
+            s.last_use = stamp;
+            p->lru_in(sids[i]);
+        }
+    }
+    p->stats.free_blocks -= need;
+    p->stats.used_blocks += need;
+    p->stats.bytes_unpacked += fetched * p->token_bytes;
+    p->stats.bytes_appended += static_cast<int64_t>(B) * p->token_bytes;
+    p->stats.appends += B;
+    if (p->host_only) return KV_OK;
+    return gather_batch(p, sids, B, block_tables, max_blocks, seq_lens, st);
 }
 
 int kv_pool_shuffle_free(kv_pool *p, uint64_t seed) {

@@ -37,7 +37,8 @@ EXPORTS = [
     "session_info", "session_block_table", "kv_pool_batch_tables", "kv_pool_shuffle_free",
     "kv_pool_free_list", "kv_pool_get_stats", "kv_pool_check_device",
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
-    "decode_attention_ex", "kv_pool_set_migration_limit",
+    "decode_attention_ex", "kv_pool_set_migration_limit", "kv_pool_batch_reserve",
+    "decode_append_attention",
 ]
 
 KV_DECODE_OVERLAP_PREVIOUS = 1
@@ -92,6 +93,8 @@ def _load():
         "session_create_paused": [p, i64, i64, C.POINTER(i32)],
         "session_destroy": [p, i32],
         "session_append": [p, i32, p, p, i32, p],
+        "kv_pool_batch_reserve": [p, p, i32, p, i32, p, p],
+        "decode_append_attention": [p, i32, p, p, p, p, p, i32, i32, C.c_float, p, C.c_uint32, p],
         "decode_attention": [p, i32, p, p, p, i32, i32, C.c_float, p, p],
         "decode_attention_ex": [p, i32, p, p, p, i32, i32, C.c_float, p, C.c_uint32, p],
         "session_pause": [p, i32, p],
@@ -191,6 +194,17 @@ def session_append(pool: int, sid: int, k, v, n: int, stream=None) -> None:
     _check(lib.session_append(pool, sid, _addr(k), _addr(v), n, _stream(stream)), "session_append")
 
 
+
+
+def decode_append_attention(pool: int, layer: int, q, k_new, v_new, block_tables, seq_lens, B: int,
+                            max_blocks: int, scale: float, out, flags: int = 0,
+                            stream=None) -> None:
+    _check(lib.decode_append_attention(pool, layer, _addr(q), _addr(k_new), _addr(v_new),
+                                       _addr(block_tables), _addr(seq_lens), B, max_blocks, scale,
+                                       _addr(out), flags, _stream(stream)),
+           "decode_append_attention")
+
+
 def decode_attention(pool: int, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
                      scale: float, out, stream=None) -> None:
     _check(lib.decode_attention(pool, layer, _addr(q), _addr(block_tables), _addr(seq_lens), B,
@@ -238,6 +252,13 @@ def kv_pool_batch_tables(pool: int, sids, block_tables, max_blocks: int, seq_len
     arr = (C.c_int32 * len(sids))(*sids)
     _check(lib.kv_pool_batch_tables(pool, arr, len(sids), _addr(block_tables), max_blocks,
                                     _addr(seq_lens), _stream(stream)), "kv_pool_batch_tables")
+
+
+def kv_pool_batch_reserve(pool: int, sids, block_tables, max_blocks: int, seq_lens,
+                          stream=None) -> None:
+    arr = (C.c_int32 * len(sids))(*sids)
+    _check(lib.kv_pool_batch_reserve(pool, arr, len(sids), _addr(block_tables), max_blocks,
+                                     _addr(seq_lens), _stream(stream)), "kv_pool_batch_reserve")
 
 
 def kv_pool_shuffle_free(pool: int, seed: int) -> None:

@@ -50,6 +50,7 @@ class TraceConfig:
     seed: int = 0
     lru: bool = False                # block residency with LRU write-on-evict
     admit_lead: int = 1              # steps between a resume and the session's first decode
+    fused_append: bool = True        # step token written by the decode kernel itself
 
 
 @dataclass
@@ -82,14 +83,19 @@ class TraceDriver:
 
     gpu=False: host-logic-only pool, no CUDA; records the peak sizes.
     gpu=True : real pool; `kv_source(sid, t0, t1)` returns device bf16 K and V
-    [L][t1-t0][Hkv][D] for the tokens appended at positions t0..t1-1.
+    [L][t1-t0][Hkv][D] for the tokens appended at positions t0..t1-1. With
+    cfg.fused_append each step's token goes through kv_pool_batch_reserve and
+    decode_append_attention; `kv_step_source(sids, positions)` may supply the
+    batch's K and V [L][B][Hkv][D] at once (else kv_source rows are stacked).
     """
 
     def __init__(self, cfg: TraceConfig, pool: int, trace: list[SessionTrace], gpu: bool,
                  kv_source=None, q=None, out=None, decode_stream=None, mig_stream=None,
-                 tables=None, seq_lens=None, max_blocks: int = 0, on_step=None):
+                 tables=None, seq_lens=None, max_blocks: int = 0, on_step=None,
+                 kv_step_source=None):
         self.cfg, self.pool, self.trace, self.gpu = cfg, pool, trace, gpu
         self.kv_source = kv_source
+        self.kv_step_source = kv_step_source
         self.q, self.out = q, out
         self.dstream, self.mstream = decode_stream, mig_stream
         self.tables, self.seq_lens, self.max_blocks = tables, seq_lens, max_blocks
@@ -143,6 +149,17 @@ class TraceDriver:
             kvtier.session_append(self.pool, sid, None, None, n, None)
         self.tokens[i] += n
         self.peak_tokens[i] = max(self.peak_tokens[i], self.tokens[i])
+
+    def _step_kv(self, members):
+        """K and V [L][B][Hkv][D] of the step's new token of each member."""
+        sids = [self.sids[i] for i in members]
+        pos = [self.tokens[i] for i in members]
+        if self.kv_step_source is not None:
+            return self.kv_step_source(sids, pos)
+        torch = self._torch
+        rows = [self.kv_source(sid, t, t + 1) for sid, t in zip(sids, pos)]
+        return (torch.cat([r[0] for r in rows], dim=1).contiguous(),
+                torch.cat([r[1] for r in rows], dim=1).contiguous())
 
     # ------------------------------------------------------------------- step
     def step(self, k: int) -> None:
@@ -201,25 +218,46 @@ class TraceDriver:
                     ev = self.admit_ev.pop(i, None)
                     if ev is not None:
                         self.dstream.wait_event(ev)
-            for i in members:                 # this step's token (path 3)
-                self._append(i, 1, self.dstream if self.gpu else None)
+            sids = [self.sids[i] for i in members]
+            B = len(sids)
+            if cfg.fused_append:             # this step's token (path 3) comes with the decode
+                if self.gpu:
+                    with self._torch.cuda.stream(self.dstream):
+                        k_new, v_new = self._step_kv(members)
+                    kvtier.kv_pool_batch_reserve(self.pool, sids, self.tables, self.max_blocks,
+                                                 self.seq_lens, self.dstream)
+                else:
+                    kvtier.kv_pool_batch_reserve(self.pool, sids, None, 1 << 20, None, None)
+                for i in members:
+                    self.tokens[i] += 1
+                    self.peak_tokens[i] = max(self.peak_tokens[i], self.tokens[i])
+            else:
+                for i in members:             # this step's token (path 3)
+                    self._append(i, 1, self.dstream if self.gpu else None)
+                if not self.gpu and cfg.lru:     # recency and spilled-block fetches
+                    kvtier.kv_pool_batch_tables(self.pool, sids, None, 1 << 20, None, None)
+                if self.gpu:
+                    kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
+                                                self.seq_lens, self.dstream)
             self.counts["appended_tokens"] += len(members)
             blocks = sum(-(-self.tokens[i] // cfg.block_tokens)
                          for i in self.active + [i for _, i in self.joining])
             self.peak_blocks = max(self.peak_blocks, blocks)
-            sids = [self.sids[i] for i in members]
-            if not self.gpu and cfg.lru:     # recency and spilled-block fetches
-                kvtier.kv_pool_batch_tables(self.pool, sids, None, 1 << 20, None, None)
             if self.gpu:
-                B = len(sids)
-                kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
-                                            self.seq_lens, self.dstream)
                 for l in range(cfg.layers):
                     # layer l > 0 follows layer l-1's call, which writes only `out`
-                    kvtier.decode_attention_ex(
-                        self.pool, l, self.q[l], self.tables, self.seq_lens, B, self.max_blocks,
-                        1 / math.sqrt(128), self.out[l],
-                        kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 else 0, self.dstream)
+                    # and (fused) layer l-1's rows of the pool
+                    flags = kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 else 0
+                    if cfg.fused_append:
+                        kvtier.decode_append_attention(
+                            self.pool, l, self.q[l], k_new[l], v_new[l], self.tables,
+                            self.seq_lens, B, self.max_blocks, 1 / math.sqrt(128), self.out[l],
+                            flags, self.dstream)
+                    else:
+                        kvtier.decode_attention_ex(
+                            self.pool, l, self.q[l], self.tables, self.seq_lens, B,
+                            self.max_blocks, 1 / math.sqrt(128), self.out[l], flags,
+                            self.dstream)
                 end.record(self.dstream)
                 self.last_decode_ev = end
                 self.step_events.append((start, end, B, sum(self.tokens[i] for i in members)))

@@ -63,7 +63,7 @@ def test_random_calls_keep_invariants(kv, lru, seed):
     sids = []
     ok = errs = 0
     for _ in range(1500):
-        op = rnd.randrange(9)
+        op = rnd.randrange(10)
         sid = rnd.choice(sids + [-1, 99, rnd.randrange(-3, 9)]) if rnd.random() < 0.9 and sids \
             else rnd.randrange(-3, 9)
         try:
@@ -93,6 +93,10 @@ def test_random_calls_keep_invariants(kv, lru, seed):
                 kv.session_info(pool, sid)
             elif op == 8:
                 kv.kv_pool_set_migration_limit(pool, rnd.choice([-1, 0, 64]))
+            elif op == 9:
+                batch = [rnd.choice(sids + [-1, 77]) if sids else -1
+                         for _ in range(rnd.randint(1, 3))]
+                kv.kv_pool_batch_reserve(pool, batch, None, rnd.choice([0, 1, 64]), None)
             ok += 1
         except kv.KVError as e:
             assert e.code in CODES, (op, e)
@@ -112,6 +116,12 @@ def test_decode_flags_and_arguments_rejected(kv):
     with pytest.raises(kv.KVError) as e:
         kv.kv_pool_set_migration_limit(pool, -5)
     assert e.value.code == kv.KV_ERR_INVALID_ARG
+    for kn, vn, code in ((None, 256, kv.KV_ERR_INVALID_ARG), (256, None, kv.KV_ERR_INVALID_ARG),
+                         (264, 256, kv.KV_ERR_INVALID_ARG),       # not 16-byte aligned
+                         (256, 512, kv.KV_ERR_BAD_STATE)):        # host-logic pool: no decode
+        with pytest.raises(kv.KVError) as e:
+            kv.decode_append_attention(pool, 0, 1024, kn, vn, 2048, 4096, 1, 1, 1.0, 8192)
+        assert e.value.code == code
     kv.kv_pool_destroy(pool)
     with pytest.raises(kv.KVError) as e:              # no-alloc path: bad shapes, before any CUDA call
         kv.decode_attention_noalloc(kv.make_config(num_layers=2, num_hot_blocks=8, head_dim=64,

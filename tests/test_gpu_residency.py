@@ -26,7 +26,10 @@ def bits(t):
     return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
 
 
-def test_residency_random_sequence(cuda_dev):
+@pytest.mark.parametrize("fused", [False, True])
+def test_residency_random_sequence(cuda_dev, fused):
+    """fused: decode batches take their step token with the decode
+    (kv_pool_batch_reserve + decode_append_attention, all layers)."""
     import __graft_entry__
     __graft_entry__.build()
     from paper_2609_25782_gb300 import Pool, kvtier
@@ -91,19 +94,37 @@ def test_residency_random_sequence(cuda_dev):
             o.pause(sid)
             pool.session_pause(sid, st)
         else:
-            batch = [x for x in live if o.s[x].state == "active" and T[x] > 0]
+            batch = [x for x in live if o.s[x].state == "active" and
+                     (T[x] < cap if fused else T[x] > 0)]
             batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 4)))
             if not batch:
                 continue
             try:
-                o.batch(batch)
+                o.batch_reserve(batch) if fused else o.batch(batch)
             except NoHotBlocks:
+                with pytest.raises(kvtier.KVError):
+                    (pool.batch_reserve if fused else pool.batch_tables)(batch, tables, mb, slens, st)
                 continue
-            pool.batch_tables(batch, tables, mb, slens, st)
             with torch.cuda.stream(st):
                 out = torch.empty(L, len(batch), Hq, D, dtype=torch.float32, device=cuda_dev)
-                pool.decode_attention(-1, q[:, :len(batch)].contiguous(), tables, slens, len(batch),
-                                      mb, 1 / math.sqrt(D), out, st)
+                qb = q[:, :len(batch)].contiguous()
+                if fused:
+                    ks, vs = [], []
+                    for x in batch:
+                        k, v = synth.kv_logical_torch(seed, x, range(L), Hkv, D, T[x], T[x] + 1,
+                                                      cuda_dev)
+                        ks.append(k[:, :, 0])
+                        vs.append(v[:, :, 0])
+                    kn, vn = torch.stack(ks, 1).contiguous(), torch.stack(vs, 1).contiguous()
+                    pool.batch_reserve(batch, tables, mb, slens, st)
+                    pool.decode_append_attention(-1, qb, kn, vn, tables, slens, len(batch), mb,
+                                                 1 / math.sqrt(D), out, st)
+                    for x in batch:
+                        T[x] += 1
+                else:
+                    pool.batch_tables(batch, tables, mb, slens, st)
+                    pool.decode_attention(-1, qb, tables, slens, len(batch), mb, 1 / math.sqrt(D),
+                                          out, st)
             torch.cuda.synchronize()
             rows = np.full((len(batch), mb), -1, dtype=np.int32)
             for i, x in enumerate(batch):

@@ -123,6 +123,50 @@ def test_no_pinning_spills_instead_of_failing():
         o.batch([0, 1])        # 9 blocks can never fit in 8
 
 
+def test_batch_reserve_hand_worked():
+    o = ResidencyOracle(6, BT, seed=7, token_bytes=TB)
+    start = list(o.fl.contents())
+    o.create(0, 1000)
+    o.append(0, 32)            # A: 2 full blocks
+    o.create(1, 1000)
+    o.append(1, 20)            # B: 2 blocks, tail holds 4 tokens
+    o.create(2, 1000)
+    o.append(2, 20)            # C: 2 blocks; pool full
+    o.pause(2)
+    c_row = o.row(2)
+    o.batch_reserve([0, 1])    # A's tail is full: one block, taken from C's block 0 (LRU)
+    assert o.row(2) == [-1, c_row[1]]
+    assert o.row(0) == [start[5], start[4], c_row[0]]
+    assert o.s[0].T == 33 and o.s[1].T == 21
+    assert o.stats["bytes_packed"] == 16 * TB and o.stats["blocks_evicted"] == 1
+    assert o.stats["bytes_appended"] == (32 + 20 + 20 + 2) * TB
+    o.resume(2)                # C's block 0 back: evicts from the least recent of A, B
+    o.batch_reserve([2])       # C at 21 tokens: no new block
+    assert o.s[2].T == 21 and len(o.row(2)) == 2
+    with pytest.raises(AssertionError):
+        o.batch_reserve([0, 0])
+
+
+def test_batch_reserve_equals_appends_then_batch_without_pressure():
+    """With free blocks to spare, reserving a step's tokens for a batch is
+    one-token appends in batch order followed by batching them."""
+    a = ResidencyOracle(200, BT, seed=9, token_bytes=TB)
+    b = ResidencyOracle(200, BT, seed=9, token_bytes=TB)
+    rnd = random.Random(3)
+    for o in (a, b):
+        for sid in range(5):
+            o.create(sid, 10_000)
+    for step in range(120):
+        batch = rnd.sample(range(5), k=rnd.randint(1, 5))
+        a.batch_reserve(batch)
+        for sid in batch:
+            b.append(sid, 1)
+        b.batch(batch)
+        assert [a.row(s) for s in range(5)] == [b.row(s) for s in range(5)]
+        assert list(a.fl.contents()) == list(b.fl.contents())
+    assert a.stats == b.stats
+
+
 # ------------------------------------------------ library vs oracle
 
 @pytest.fixture(scope="module")
@@ -161,7 +205,7 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
     pool, tb = lib_pool(kv, nb, seed)
     o = ResidencyOracle(nb, BT, seed=seed, token_bytes=tb)
     live = []
-    fails = 0
+    fails = reserved = 0
     for step in range(500):
         r = rnd.random()
         try:
@@ -216,7 +260,7 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
                 elif r < 0.75:
                     o.pause(sid)
                     kv.session_pause(pool, sid, None)
-                else:
+                elif r < 0.87:
                     batch = [x for x in live if o.s[x].state == "active" and o.s[x].T > 0]
                     batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 3)))
                     if not batch:
@@ -232,9 +276,71 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
                     except kv.KVError as e:
                         assert e.code == exp
                         fails += 1
+                else:               # a fused decode step's token for each member
+                    batch = [x for x in live if o.s[x].state == "active" and o.s[x].T < 400]
+                    batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 3)))
+                    if not batch:
+                        continue
+                    exp = None
+                    try:
+                        o.batch_reserve(batch)
+                    except NoHotBlocks:
+                        exp = kv.KV_ERR_NO_HOT_BLOCKS
+                    try:
+                        kv.kv_pool_batch_reserve(pool, batch, None, 64, None)
+                        assert exp is None
+                        reserved += 1
+                    except kv.KVError as e:
+                        assert e.code == exp
+                        fails += 1
         finally:
             pass
         compare(kv, pool, o, live)
     st = kv.kv_pool_get_stats(pool)
-    assert st["blocks_evicted"] > 20 and st["resume_blocks_missed"] > 0
+    assert st["blocks_evicted"] > 20 and st["resume_blocks_missed"] > 0 and reserved > 10
     kv.kv_pool_destroy(pool)
+
+
+def test_batch_reserve_simple_mode_equals_one_token_appends(kv):
+    """Without residency, a batch reservation pops exactly the blocks that
+    one-token appends in batch order would, and fails atomically."""
+    def pool():
+        cfg = kv.make_config(num_layers=1, num_hot_blocks=40, block_tokens=BT, alloc_seed=5,
+                             max_sessions=6, max_context=4096, max_batch=8,
+                             cold_bytes=6 * 4096 * 2 * 4 * 128 * 2,
+                             flags=kv.KV_POOL_HOST_LOGIC_ONLY)
+        p = kv.kv_pool_create(cfg)
+        for _ in range(5):
+            kv.session_create(p, 300)
+        return p
+    a, b = pool(), pool()
+    rnd = random.Random(11)
+    for step in range(150):
+        batch = rnd.sample(range(5), k=rnd.randint(1, 5))
+        if any(kv.session_info(a, s).tokens >= 300 for s in batch):
+            continue
+        kv.kv_pool_batch_reserve(a, batch, None, 64, None)
+        for sid in batch:
+            kv.session_append(b, sid, None, None, 1, None)
+        assert [kv.session_block_table(a, s) for s in range(5)] == \
+            [kv.session_block_table(b, s) for s in range(5)]
+        assert kv.kv_pool_free_list(a) == kv.kv_pool_free_list(b)
+    sa, sb = kv.kv_pool_get_stats(a), kv.kv_pool_get_stats(b)
+    assert sa == sb
+    # errors leave everything as it was
+    before = ([kv.session_block_table(a, s) for s in range(5)], kv.kv_pool_free_list(a))
+    for bad, code in (([0, 0], kv.KV_ERR_INVALID_ARG), ([0, 9], kv.KV_ERR_INVALID_ARG)):
+        with pytest.raises(kv.KVError) as e:
+            kv.kv_pool_batch_reserve(a, bad, None, 64, None)
+        assert e.value.code == code
+    assert before == ([kv.session_block_table(a, s) for s in range(5)], kv.kv_pool_free_list(a))
+    kv.session_pause(a, 1, None)
+    before = ([kv.session_block_table(a, s) for s in range(5)], kv.kv_pool_free_list(a),
+              kv.session_info(a, 0).tokens)
+    with pytest.raises(kv.KVError) as e:
+        kv.kv_pool_batch_reserve(a, [0, 1], None, 64, None)   # member 0 is fine, 1 is paused
+    assert e.value.code == kv.KV_ERR_BAD_STATE
+    assert before == ([kv.session_block_table(a, s) for s in range(5)], kv.kv_pool_free_list(a),
+                      kv.session_info(a, 0).tokens)
+    kv.kv_pool_destroy(a)
+    kv.kv_pool_destroy(b)
