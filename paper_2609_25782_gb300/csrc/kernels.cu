@@ -647,6 +647,9 @@ __global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__
 // K5: one warp per (layer, token): the token's K and V rows for all kv-heads
 // are 2 x Hkv*256 contiguous bytes in the source; each 256-byte head row goes
 // to its (layer, K|V, head) run of the tail block.
+// One warp per (layer, token) item, items layer-major so that consecutive
+// warps read k and v sequentially. A lane issues all of its 16-byte loads of
+// the item (K and V rows of every kv-head) before its first store.
 __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
     const Shape sh = a.s;
     const int items = sh.L * a.n;
@@ -657,21 +660,31 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
         const int l = it / a.n;
         const int i = it - l * a.n;
         const int64_t t = a.pos0 + i;
-        const int blk = a.table[t / sh.bt];
-        if (blk < 0 || blk >= sh.num_blocks) {
-            if (lane == 0) atomicOr(a.err, kErrBadBlock);
-            continue;
-        }
-        const int slot = static_cast<int>(t % sh.bt);
         const int64_t src_off = static_cast<int64_t>(it) * sh.Hkv * kRowBytes;
-        const int64_t run0 = (static_cast<int64_t>(blk) * sh.L + l) * 2 * sh.Hkv;
-        for (int u = lane; u < 2 * units; u += 32) {
-            const int kv = u >= units;
-            const int uu = u - kv * units;
-            const int g = uu >> 4;                  // 16 units per head row
-            const uint4 v = reinterpret_cast<const uint4 *>((kv ? a.v : a.k) + src_off)[uu];
-            uint8_t *dst = a.hot + (((run0 + kv * sh.Hkv + g) * sh.bt + slot) * kRowBytes);
-            reinterpret_cast<uint4 *>(dst)[uu & 15] = v;
+        const uint4 *ks = reinterpret_cast<const uint4 *>(a.k + src_off);
+        const uint4 *vs = reinterpret_cast<const uint4 *>(a.v + src_off);
+        const int blk = a.table[t / sh.bt];
+        const bool ok = blk >= 0 && blk < sh.num_blocks;
+        if (!ok && lane == 0) atomicOr(a.err, kErrBadBlock);
+        // Unit u = (kv * Hkv + g) * 16 + c lands in run (kv, g), row `slot`.
+        const int slot = static_cast<int>(t % sh.bt);
+        uint8_t *base = a.hot + ((static_cast<int64_t>(ok ? blk : 0) * sh.L + l) * 2 * sh.Hkv *
+                                     sh.bt + slot) * kRowBytes;
+        const int64_t run_bytes = static_cast<int64_t>(sh.bt) * kRowBytes;
+        for (int u0 = 0; u0 < 2 * units; u0 += 32 * KVT_MIG_UNROLL) {
+            uint4 v[KVT_MIG_UNROLL];
+#pragma unroll
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < 2 * units) v[k] = ld_stream(u < units ? ks + u : vs + (u - units));
+            }
+            if (!ok) continue;
+#pragma unroll
+            for (int k = 0; k < KVT_MIG_UNROLL; ++k) {
+                const int u = u0 + k * 32 + lane;
+                if (u < 2 * units)
+                    st_out(reinterpret_cast<uint4 *>(base + (u >> 4) * run_bytes) + (u & 15), v[k]);
+            }
         }
     }
 }
