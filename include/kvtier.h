@@ -126,8 +126,10 @@ typedef struct kv_pool_stats {
     int64_t cold_bytes_used;
     int64_t bytes_unpacked;   /* image bytes copied cold -> hot (path 2)   */
     int64_t bytes_packed;     /* image bytes copied hot -> cold (path 4)   */
-    int64_t bytes_appended;   /* KV bytes written by session_append        */
-    int64_t resumes, pauses, appends, decodes;
+    int64_t bytes_appended;   /* KV bytes of tokens added by session_append
+                               * and kv_pool_batch_reserve                  */
+    int64_t resumes, pauses, appends, decodes; /* appends: calls, plus one per
+                                                * reserved batch member    */
     int64_t blocks_evicted;       /* residency mode: blocks evicted            */
     int64_t resume_blocks_hit;    /* residency mode: still hot at resume       */
     int64_t resume_blocks_missed; /* residency mode: fetched at resume         */
