@@ -35,11 +35,21 @@ namespace {
 #define KVT_STAGES 2   // 4 warps x 2 x 8 KiB: 3 CTAs (24 tiles in flight) per SM
 #endif
 constexpr int kDecodeWarps = KVT_DECODE_WARPS;
-constexpr int kStages = KVT_STAGES;        // tiles in flight per warp
 constexpr int kCombineWarps = 4;
 constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
 constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
-constexpr int kDecodeSmem = kDecodeWarps * kStages * kTileBytes + 1024 + 256;
+// Ring depths (tiles in flight per warp) by how many CTAs share an SM: a
+// grid that fills every SM three times over runs 3 CTAs of KVT_STAGES slots
+// per SM; smaller grids get deeper rings so each SM still keeps ~24 tiles
+// in flight. The depth changes only the prefetch distance, never which warp
+// takes which tile, so all variants give bit-identical results.
+constexpr int kStagesFull = KVT_STAGES;    // 3 CTAs per SM
+constexpr int kStagesHalf = 3;             // 2 CTAs per SM
+constexpr int kStagesOne = 6;              // 1 CTA per SM
+__host__ __device__ constexpr int decode_smem(int stages) {
+    return kDecodeWarps * stages * kTileBytes + 1024 + 256;   // rings, alignment, barriers
+}
+static_assert(kDecodeWarps * kStagesOne * 8 <= 256, "mbarriers must fit their 256-byte area");
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;   // 2 s
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -151,6 +161,7 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 // The four warps' states merge in shared memory in warp order; a one-split
 // session writes its normalised output, others write (m, l, acc) partials.
 // ---------------------------------------------------------------------------
+template <int kStages>
 __global__ void __launch_bounds__(kDecodeWarps * 32)
     decode_split_kernel(const __grid_constant__ CUtensorMap map, const DecodeArgs a) {
     extern __shared__ uint8_t smem_raw[];
@@ -733,12 +744,22 @@ bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const
 }
 
 cudaError_t prepare_kernels() {
-    return cudaFuncSetAttribute(decode_split_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kDecodeSmem);
+    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<kStagesFull>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         decode_smem(kStagesFull));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(decode_split_kernel<kStagesHalf>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 decode_smem(kStagesHalf));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(decode_split_kernel<kStagesOne>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 decode_smem(kStagesOne));
+    return e;
 }
 
-cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st,
-                          bool overlap_previous) {
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_sms,
+                          cudaStream_t st, bool overlap_previous) {
     // Every session of the batch has T <= max_blocks * bt, so its splits fit.
     const int splits = max_splits_for(static_cast<int64_t>(a.max_blocks) * a.s.bt);
     if (splits > a.max_splits) return cudaErrorInvalidValue;
@@ -749,12 +770,27 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStrea
     cudaLaunchConfig_t c1 = {};
     c1.gridDim = dim3(splits, a.s.Hkv, a.nlayers * a.B);
     c1.blockDim = dim3(kDecodeWarps * 32);
-    c1.dynamicSmemBytes = kDecodeSmem;
     c1.stream = st;
     c1.attrs = overlap_previous ? attr : nullptr;
     c1.numAttrs = overlap_previous ? 1 : 0;
-    cudaError_t e = cudaLaunchKernelEx(&c1, decode_split_kernel, map, a);
+    // CTAs of the grid (an upper bound: splits past a session's own count
+    // exit at once) against the SMs decide the ring depth.
+    const int64_t ctas = static_cast<int64_t>(splits) * a.s.Hkv * a.nlayers * a.B;
+    cudaError_t e;
+    if (ctas <= num_sms) {
+        c1.dynamicSmemBytes = decode_smem(kStagesOne);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesOne>, map, a);
+    } else if (ctas <= 2 * static_cast<int64_t>(num_sms)) {
+        c1.dynamicSmemBytes = decode_smem(kStagesHalf);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesHalf>, map, a);
+    } else {
+        c1.dynamicSmemBytes = decode_smem(kStagesFull);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesFull>, map, a);
+    }
     if (e != cudaSuccess) return e;
+    // Tables at most 1 024 tokens wide: every session is one split and the
+    // split kernel has written the outputs itself.
+    if (splits == 1) return cudaSuccess;
 
     cudaLaunchConfig_t c2 = {};
     c2.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));

@@ -139,9 +139,10 @@ struct GatherArgs {
 bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why);
 cudaError_t prepare_kernels();  // per-device function attributes
 // overlap_previous: launch the split kernel as a programmatic dependent of the
-// previous kernel on the stream (see decode_attention_ex).
-cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, cudaStream_t st,
-                          bool overlap_previous);
+// previous kernel on the stream (see decode_attention_ex). num_sms sizes the
+// split kernel's tile rings to the grid.
+cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_sms,
+                          cudaStream_t st, bool overlap_previous);
 // max_ctas > 0 caps the migration grids (kv_pool_set_migration_limit).
 cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);
 cudaError_t launch_pack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);

@@ -22,6 +22,7 @@ static __device__ __align__(256) unsigned char g_decode_scratch[KV_NOALLOC_SCRAT
 
 struct DeviceScratch {
     unsigned char *ptr = nullptr;   // device address of g_decode_scratch
+    int num_sms = 1;
     bool ready = false;
 };
 DeviceScratch g_dev[kMaxDevices];
@@ -34,8 +35,8 @@ int fail(int code, const char *msg) {
 
 // Per-device set-up, run by the first call on each device with that device
 // current: the array's device address (the host-side symbol is only a
-// stand-in) and the decode kernel's shared-memory attribute.
-int setup_device(int dev, unsigned char **ptr) {
+// stand-in), the decode kernels' shared-memory attributes and the SM count.
+int setup_device(int dev, unsigned char **ptr, int *num_sms) {
     std::lock_guard<std::mutex> lk(g_mu);
     DeviceScratch &d = g_dev[dev];
     if (!d.ready) {
@@ -44,10 +45,13 @@ int setup_device(int dev, unsigned char **ptr) {
             return fail(KV_ERR_CUDA, "decode_attention_noalloc: cudaGetSymbolAddress failed");
         if (kvt::prepare_kernels() != cudaSuccess)
             return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel attribute set-up failed");
+        if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return fail(KV_ERR_CUDA, "decode_attention_noalloc: SM count query failed");
         d.ptr = static_cast<unsigned char *>(p);
         d.ready = true;
     }
     *ptr = d.ptr;
+    *num_sms = d.num_sms;
     return KV_OK;
 }
 
@@ -102,7 +106,8 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     } restore{prev, c.device};
 
     unsigned char *scratch = nullptr;
-    int rc = setup_device(c.device, &scratch);
+    int num_sms = 1;
+    int rc = setup_device(c.device, &scratch, &num_sms);
     if (rc) return rc;
     CUtensorMap map;
     const char *why = nullptr;
@@ -133,7 +138,7 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     a.k_new = a.v_new = nullptr;
     a.hot = nullptr;
     a.s = kvt::Shape{c.num_layers, c.num_q_heads, c.num_kv_heads, c.block_tokens, c.num_hot_blocks};
-    if (kvt::launch_decode(map, a, st, false) != cudaSuccess)
+    if (kvt::launch_decode(map, a, num_sms, st, false) != cudaSuccess)
         return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel launch failed");
     return KV_OK;
 }

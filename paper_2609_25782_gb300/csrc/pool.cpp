@@ -811,7 +811,7 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     const bool overlap = (flags & KV_DECODE_OVERLAP_PREVIOUS) != 0;
-    int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, st, overlap); });
+    int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, p->num_sms, st, overlap); });
     if (rc) return rc;
     p->stats.decodes += 1;
     return KV_OK;

@@ -147,11 +147,14 @@ def queries_np(seed: int, sess_ids, layers, num_q_heads: int, head_dim: int):
 def session_lengths(seed: int, n: int, lo: int, hi: int, block_tokens: int = 16,
                     need_partial: bool = True) -> np.ndarray:
     """n integer lengths uniform on [lo, hi]; with need_partial, at least one
-    length is not a multiple of block_tokens."""
+    length is not a multiple of block_tokens when [lo, hi] holds one."""
     rng = np.random.Generator(np.random.PCG64(seed))
     t = rng.integers(lo, hi + 1, size=n).astype(np.int64)
     if need_partial and n > 0 and np.all(t % block_tokens == 0):
-        t[0] = t[0] - 1 if t[0] - 1 >= lo else t[0] + 1
+        if t[0] - 1 >= lo:
+            t[0] -= 1
+        elif t[0] + 1 <= hi:
+            t[0] += 1
     return t
 
 

@@ -139,6 +139,28 @@ def test_decode_independent_of_batch_and_placement(pkg):
     assert np.array_equal(moved, full)
 
 
+def test_ring_depths_bit_identical(pkg):
+    """The split kernel's tile-ring depth follows the size of the grid (6, 3
+    or 2 tiles in flight per warp for 1, 2 or 3 CTAs per SM). It changes only
+    how far ahead tiles are fetched, so all three must give the same bits."""
+    lens = [5000, 3001, 777]
+    L = 16
+    pool, sess, tables, q = direct_case(pkg, lens, L=L, seed=4, max_batch=L * len(lens))
+    wide = np.pad(tables, ((0, 0), (0, 2048 - tables.shape[1])), constant_values=-1)
+    # per layer, 313-block tables: 5 splits x 4 kv-heads x 3 rows = 60 CTAs (6-deep rings);
+    # per layer, tables 2048 blocks wide: 16 x 4 x 3 = 192 CTAs (3-deep);
+    # all 16 layers in one call: 5 x 4 x 48 = 960 CTAs (2-deep)
+    narrow = np.concatenate([gpu_decode(pool, l, q, tables, lens) for l in range(L)])
+    padded = np.concatenate([gpu_decode(pool, l, q, wide, lens) for l in range(L)])
+    whole = gpu_decode(pool, -1, q, tables, lens)
+    assert np.array_equal(narrow.view(np.int64), padded.view(np.int64))
+    assert np.array_equal(narrow.view(np.int64), whole.view(np.int64))
+    ref = oracle.paged_decode(host_hot(pool, 4, sess, lens, tables), q.cpu().view(torch.int16)
+                              .numpy().view(np.uint16), tables, lens, 1 / math.sqrt(128), 32)
+    assert scaled_err(narrow, ref) <= TOL
+    assert pool.check_device() == 0
+
+
 def test_overlapped_calls_bit_identical(pkg):
     """Per-layer calls launched with KV_DECODE_OVERLAP_PREVIOUS (each one
     overlapping the previous call's end) give the same bits as serialised

@@ -287,3 +287,14 @@ def test_free_list_pop_push_contract():
     assert list(fl.contents()) == list(start[:7]) + list(got)
     with pytest.raises(MemoryError):
         fl.pop(11)
+
+
+def test_session_lengths_stay_in_range():
+    """Lengths are draws on [lo, hi]; one is made ragged (not a multiple of
+    the block size) only when [lo, hi] holds such a length."""
+    for seed, n, lo, hi in [(0, 1, 65536, 65536), (1, 3, 16, 16), (2, 32, 8192, 32768),
+                            (3, 4, 64, 65), (4, 8, 1, 2048), (5, 2, 32, 47)]:
+        t = synth.session_lengths(seed, n, lo, hi, 16)
+        assert len(t) == n and t.min() >= lo and t.max() <= hi
+        if any(x % 16 for x in range(lo, hi + 1)):
+            assert any(int(x) % 16 for x in t)
