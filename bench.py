@@ -335,6 +335,13 @@ def run_migration(args, rank):
     torch.cuda.synchronize()
     img_bytes = T * TOKEN_BYTES
 
+    def gate(stream):
+        """Keep the stream busy (a short spin) while the host enqueues the timed
+        calls, so the start event fires with their launches already queued and
+        the interval is device time, not host launch latency."""
+        with torch.cuda.stream(stream):
+            torch.cuda._sleep(1_000_000)
+
     def burst(reps):
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(n_sess)]
@@ -343,6 +350,7 @@ def run_migration(args, rank):
         tot = 0.0
         per = []
         for _ in range(reps):
+            gate(st)
             a.record(st)
             for i, s in enumerate(sids):
                 ev[i][0].record(st)
@@ -358,15 +366,17 @@ def run_migration(args, rank):
 
     burst(1)
     burst_ms, per = burst(max(2, args.steps // 4))
-    alone = []
+    alone, alone_idle = [], []
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
-    for _ in range(3):
+    for rep in range(6):
+        if rep % 2 == 0:
+            gate(st)
         a.record(st)
         pool.session_resume(sids[0], st)
         b.record(st)
         torch.cuda.synchronize()
-        alone.append(a.elapsed_time(b))
+        (alone if rep % 2 == 0 else alone_idle).append(a.elapsed_time(b))
         pool.session_pause(sids[0], st)
     flags = pool.check_device()
 
@@ -383,6 +393,7 @@ def run_migration(args, rank):
         for s in fresh:
             pool.session_append(s, kk, vv, st)
         torch.cuda.synchronize()
+        gate(st)
         a.record(st)
         for s in fresh:
             pool.session_pause(s, st)
@@ -405,6 +416,7 @@ def run_migration(args, rank):
             "gbs_rw": round(unpack_rw, 1), "frac_rw": round(unpack_rw / peak, 3),
             "per_session_ms_in_burst": round(statistics.mean(per), 3),
             "per_session_ms_alone": round(statistics.median(alone), 3),
+            "per_session_ms_alone_from_idle_gpu": round(statistics.median(alone_idle), 3),
         },
         "pause_pack": {
             "sessions": n_sess, "tokens": T, "burst_ms": round(pack_ms_m, 3),
@@ -627,19 +639,26 @@ def run_sweep(args):
     for T in SWEEP_T:
         s = pool.session_create_paused(T, T)
         synth.fill_image_torch(pool.image(s), args.seed, s, L, HKV, D, T)
-        ms = []
-        for rep in range(6):
+        ms, ms_idle = [], []
+        for rep in range(12):
+            # even reps: device time (a spin keeps the stream busy while the host
+            # enqueues the resume, so the start event fires with its launches
+            # queued); odd reps: from an idle GPU, host enqueue included
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if rep % 2 == 0:
+                with torch.cuda.stream(stream):
+                    torch.cuda._sleep(1_000_000)
             a.record(stream)
             pool.session_resume(s, stream)
             b.record(stream)
             torch.cuda.synchronize()
-            if rep >= 2:
-                ms.append(a.elapsed_time(b))
+            if rep >= 4:
+                (ms if rep % 2 == 0 else ms_idle).append(a.elapsed_time(b))
             pool.session_pause(s, stream)
         m = statistics.median(ms)
         rw = 2 * T * TOKEN_BYTES / (m * 1e-3) / 1e9
-        resume.append({"T": T, "ms": round(m, 4), "gbs_rw": round(rw, 1), "frac": round(rw / peak, 3)})
+        resume.append({"T": T, "ms": round(m, 4), "gbs_rw": round(rw, 1), "frac": round(rw / peak, 3),
+                       "ms_from_idle_gpu": round(statistics.median(ms_idle), 4)})
         pool.session_destroy(s)
     pool.close()
     return {"decode": points, "resume": resume, "peak_gbs": peak}
