@@ -300,10 +300,16 @@ int kv_pool_free_list(kv_pool *pool, int32_t *host_out, int64_t cap, int64_t *n)
 
 int kv_pool_get_stats(kv_pool *pool, kv_pool_stats *out);
 
+/* Bits of the device flag word that kernels set when their own checks fire. */
+#define KV_DEVICE_BAD_BLOCK 1   /* a block id outside the pool (access skipped)     */
+#define KV_DEVICE_BAD_LENGTH 2  /* seq_len < 1 or past its table row (row skipped) */
+#define KV_DEVICE_TIMEOUT 4     /* a tile wait gave up after 2 s (output undefined) */
+
 /* Synchronise the device and read the flags that kernels set when their own
  * bounds checks fire (a block id outside the pool, a length past a table
  * row, a wait that timed out); clears them. *flags = 0 means clean; a
- * non-zero value makes the call return KV_ERR_DEVICE_CHECK. */
+ * non-zero value (KV_DEVICE_* bits) makes the call return
+ * KV_ERR_DEVICE_CHECK. */
 int kv_pool_check_device(kv_pool *pool, int32_t *flags);
 
 /* Cap the migration kernels (resume-unpack, pause-pack, evictions) at
@@ -317,6 +323,16 @@ int kv_pool_set_migration_limit(kv_pool *pool, int32_t max_ctas);
  * CUDA error) so tests can check that failing calls change nothing;
  * n <= 0 disarms. */
 int kv_pool_inject_cuda_failure(kv_pool *pool, int32_t n);
+
+/* Test hook for the decode kernel's bounded waits: with on != 0, the next
+ * decode call makes warp 0 of one CTA (split 0, kv-head 0, first row) expect
+ * 16 bytes more than its first tile copy delivers. Every copy still lands;
+ * that one wait runs out after its 2 s limit, the kernel sets
+ * KV_DEVICE_TIMEOUT, waits (bounded) for the warp's other copies and
+ * finishes. That call's output for the row is undefined; the CUDA context
+ * stays usable and kv_pool_check_device reports the flag. Disarms itself
+ * after one call. */
+int kv_pool_inject_decode_timeout(kv_pool *pool, int32_t on);
 
 /* Fixed size of the device scratch used by decode_attention_noalloc. */
 #define KV_NOALLOC_SCRATCH_BYTES (48ll << 20)

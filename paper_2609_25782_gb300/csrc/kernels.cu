@@ -221,7 +221,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         const int rowv = rowk + chunk_rows;
         const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
         const uint32_t bar = bar0 + 8 * (k % kStages);
-        mbar_expect_tx(bar, kTileBytes);
+        // inject_extra_tx (a test of the bounded wait, 0 in normal calls): this
+        // one barrier then never completes its phase, although every copy lands.
+        const bool injected = k == 0 && warp == 0 && split == 0 && g == 0 && lb == 0;
+        mbar_expect_tx(bar, kTileBytes + (injected ? a.inject_extra_tx : 0));
         tma_load_2d(slot, &map, 0, rowk, bar);
         tma_load_2d(slot + kHalfBytes, &map, 64, rowk, bar);
         tma_load_2d(slot + 2 * kHalfBytes, &map, 0, rowv, bar);

@@ -74,6 +74,7 @@ struct DecodeArgs {
     // written into its reserved pool slot as well as attended to.
     const uint16_t *k_new, *v_new;
     uint16_t *hot;            // pool base, written only when k_new is set
+    int32_t inject_extra_tx;  // test hook: extra bytes expected on one tile (0 normally)
     Shape s;
 };
 

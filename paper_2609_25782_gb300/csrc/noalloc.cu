@@ -137,6 +137,7 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     a.out_bf16 = 0;
     a.k_new = a.v_new = nullptr;
     a.hot = nullptr;
+    a.inject_extra_tx = 0;
     a.s = kvt::Shape{c.num_layers, c.num_q_heads, c.num_kv_heads, c.block_tokens, c.num_hot_blocks};
     if (kvt::launch_decode(map, a, num_sms, st, false) != cudaSuccess)
         return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel launch failed");

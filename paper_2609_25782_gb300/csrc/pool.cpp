@@ -17,6 +17,10 @@
 #include "../../include/kvtier.h"
 #include "kvt_internal.h"
 
+static_assert(KV_DEVICE_BAD_BLOCK == kvt::kErrBadBlock && KV_DEVICE_BAD_LENGTH == kvt::kErrBadLength &&
+                  KV_DEVICE_TIMEOUT == kvt::kErrTimeout,
+              "public device flag bits must match the kernels'");
+
 namespace {
 
 thread_local std::string g_last_error;
@@ -119,6 +123,7 @@ struct kv_pool {
 
     kv_pool_stats stats{};
     int32_t inject_countdown = 0;
+    bool inject_timeout = false;   // kv_pool_inject_decode_timeout, next decode only
 
     // Residency mode (KV_POOL_LRU_RESIDENCY): sessions holding hot blocks,
     // ordered by (last use, sid); the first one is the least recently used.
@@ -808,11 +813,13 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
     a.k_new = static_cast<const uint16_t *>(k_new);
     a.v_new = static_cast<const uint16_t *>(v_new);
     a.hot = static_cast<uint16_t *>(p->cfg.hot_base);
+    a.inject_extra_tx = p->inject_timeout ? 16 : 0;
     a.s = p->shape;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream_);
     const bool overlap = (flags & KV_DECODE_OVERLAP_PREVIOUS) != 0;
     int rc = p->cuda("decode launch", [&] { return kvt::launch_decode(p->tmap, a, p->num_sms, st, overlap); });
     if (rc) return rc;
+    p->inject_timeout = false;
     p->stats.decodes += 1;
     return KV_OK;
 }
@@ -1154,6 +1161,12 @@ int kv_pool_set_migration_limit(kv_pool *p, int32_t max_ctas) {
 int kv_pool_inject_cuda_failure(kv_pool *p, int32_t n) {
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     p->inject_countdown = n > 0 ? n : 0;
+    return KV_OK;
+}
+
+int kv_pool_inject_decode_timeout(kv_pool *p, int32_t on) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    p->inject_timeout = on != 0;
     return KV_OK;
 }
 

@@ -122,7 +122,12 @@ def test_decode_flags_and_arguments_rejected(kv):
         with pytest.raises(kv.KVError) as e:
             kv.decode_append_attention(pool, 0, 1024, kn, vn, 2048, 4096, 1, 1, 1.0, 8192)
         assert e.value.code == code
+    kv.kv_pool_inject_decode_timeout(pool, 1)          # armed, then disarmed: host state only
+    kv.kv_pool_inject_decode_timeout(pool, 0)
     kv.kv_pool_destroy(pool)
+    with pytest.raises(kv.KVError) as e:
+        kv.kv_pool_inject_decode_timeout(None, 1)
+    assert e.value.code == kv.KV_ERR_INVALID_ARG
     with pytest.raises(kv.KVError) as e:              # no-alloc path: bad shapes, before any CUDA call
         kv.decode_attention_noalloc(kv.make_config(num_layers=2, num_hot_blocks=8, head_dim=64,
                                                    hot_base=256), 0, 1, 1, 1, 1, 1, 1.0, 1)
