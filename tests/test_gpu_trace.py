@@ -167,3 +167,78 @@ def test_full_trace_sampled_parity(cuda_dev):
         kk, vv = synth.session_kv_np(cfg.seed, i, [l], Hkv, D, n)
         assert np.array_equal(img[0], kk[0]) and np.array_equal(img[1], vv[0])
     pool.close()
+
+
+def test_small_trace_residency_under_pressure(cuda_dev):
+    """The small trace in residency mode (LRU, write-on-evict) with a hot pool
+    of exactly the simple mode's peak: paused sessions' blocks are evicted and
+    fetched back, step tokens go through the fused decode. At sampled steps
+    the decode must match the oracle over the members' logical KV (so every
+    block fetched back holds the right bytes), and the run's counters must
+    equal the residency dry run's."""
+    import dataclasses
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool, kvtier
+    from paper_2609_25782_gb300 import trace as tr
+
+    base = tr.TraceConfig(sessions=6, t0_min=100, t0_max=700, burst_mean=8.0, pause_mean_s=0.6,
+                          append_median=40.0, append_sigma=1.0, append_max=300, active_cap=2,
+                          steps=150, dt_s=0.1, layers=2, seed=5)
+    trace = tr.generate(base)
+    simple = tr.plan(base, trace)
+    cfg = dataclasses.replace(base, lru=True)
+    nb = simple["peak_blocks"]
+    dry = tr.plan(cfg, trace, hot_blocks=nb)["stats"]
+    assert dry["blocks_evicted"] > 0 and dry["resume_blocks_missed"] > 0
+    L, Hkv, Hq, D, bt = cfg.layers, cfg.num_kv_heads, cfg.num_q_heads, 128, cfg.block_tokens
+    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=simple["cold_bytes"] + 4096,
+                max_sessions=cfg.sessions, max_batch=cfg.active_cap,
+                max_context=simple["max_context"], alloc_seed=cfg.seed, lru_residency=True)
+    for i, t in enumerate(trace):
+        sid = pool.session_create_paused(simple["caps"][i], t.t0)
+        synth.fill_image_torch(pool.image(sid), cfg.seed, sid, L, Hkv, D, t.t0)
+
+    def kv_source(sid, t0, t1):
+        k, v = synth.kv_logical_torch(cfg.seed, sid, range(L), Hkv, D, t0, t1, cuda_dev)
+        return k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+
+    q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(L), Hq, D, cuda_dev)
+    out = torch.empty(L, cfg.active_cap, Hq, D, dtype=torch.float32, device=cuda_dev)
+    max_blocks = -(-simple["max_context"] // bt)
+    tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=cuda_dev)
+    seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=cuda_dev)
+    torch.cuda.synchronize()
+    checked = []
+
+    def on_step(k, members):
+        if k % 7 != 3:
+            return
+        torch.cuda.synchronize()
+        got = out[:, :len(members)].double().cpu().numpy()
+        lens = [int(kvtier.session_info(pool.handle, m).tokens) for m in members]
+        tab = np.full((len(members), max_blocks), -1, dtype=np.int32)
+        for r, m in enumerate(members):
+            row = pool.session_block_table(m)
+            assert min(row) >= 0                   # the batch's blocks are all hot
+            tab[r, :len(row)] = row
+        hot = synth.hot_pool_np(cfg.seed, members, lens, tab, nb, L, Hkv, D, bt)
+        qh = q[:, :len(members)].contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+        ref = oracle.paged_decode(hot, qh, tab, lens, 1 / math.sqrt(D), Hq)
+        err = np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref)))
+        assert err <= TOL, f"step {k}: scaled error {err}"
+        checked.append(k)
+
+    d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
+                       decode_stream=torch.cuda.Stream(), mig_stream=torch.cuda.Stream(),
+                       tables=tables, seq_lens=seq_lens, max_blocks=max_blocks, on_step=on_step)
+    d.run()
+    torch.cuda.synchronize()
+    assert len(checked) >= 10
+    assert pool.check_device() == 0
+    st = pool.stats()
+    for key in ("bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
+                "resume_blocks_missed", "resumes", "pauses"):
+        assert st[key] == dry[key], key
+    pool.close()
