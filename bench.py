@@ -556,14 +556,48 @@ SWEEP_CAP = 120e9
 
 
 def run_sweep(args):
-    """Roofline-fraction curve: decode over (block size, batch, context) with
-    total KV <= 120 GB, per-layer launches and the all-layers launch; then the
-    resume-unpack sweep over single sessions of 1K..128K tokens."""
+    """Roofline-fraction curve: the resume-unpack sweep over single sessions of
+    1K..128K tokens, then decode over (block size, batch, context) with total
+    KV <= 120 GB, per-layer launches and the all-layers launch."""
     import torch
     import synth
     from paper_2609_25782_gb300 import Pool
     dev = torch.device("cuda", torch.cuda.current_device())
     peak, _ = hbm_peak()
+    # resume-unpack sweep (first, before the long decode sweep loads the GPU)
+    resume = []
+    Tm = max(SWEEP_T)
+    pool = Pool(num_layers=L, num_hot_blocks=Tm // 16 + 64, cold_bytes=Tm * TOKEN_BYTES * 2 + 4096,
+                max_sessions=len(SWEEP_T) + 1, max_batch=4, max_context=Tm, alloc_seed=args.seed,
+                device=dev.index)
+    stream = torch.cuda.Stream(device=dev)
+    for T in SWEEP_T:
+        s = pool.session_create_paused(T, T)
+        synth.fill_image_torch(pool.image(s), args.seed, s, L, HKV, D, T)
+        ms, ms_idle = [], []
+        for rep in range(12):
+            # even reps: device time (a spin keeps the stream busy while the host
+            # enqueues the resume, so the start event fires with its launches
+            # queued); odd reps: from an idle GPU, host enqueue included
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if rep % 2 == 0:
+                with torch.cuda.stream(stream):
+                    torch.cuda._sleep(1_000_000)
+            a.record(stream)
+            pool.session_resume(s, stream)
+            b.record(stream)
+            torch.cuda.synchronize()
+            if rep >= 4:
+                (ms if rep % 2 == 0 else ms_idle).append(a.elapsed_time(b))
+            pool.session_pause(s, stream)
+        m = statistics.median(ms)
+        rw = 2 * T * TOKEN_BYTES / (m * 1e-3) / 1e9
+        resume.append({"T": T, "ms": round(m, 4), "gbs_rw": round(rw, 1), "frac": round(rw / peak, 3),
+                       "ms_from_idle_gpu": round(statistics.median(ms_idle), 4)})
+        pool.session_destroy(s)
+    pool.close()
+    del pool
+    torch.cuda.empty_cache()
     scale = 1 / math.sqrt(D)
     points = []
     for bt in (16, 64):
@@ -629,38 +663,6 @@ def run_sweep(args):
         pool.close()
         del pool
         torch.cuda.empty_cache()
-    # resume-unpack sweep
-    resume = []
-    Tm = max(SWEEP_T)
-    pool = Pool(num_layers=L, num_hot_blocks=Tm // 16 + 64, cold_bytes=Tm * TOKEN_BYTES * 2 + 4096,
-                max_sessions=len(SWEEP_T) + 1, max_batch=4, max_context=Tm, alloc_seed=args.seed,
-                device=dev.index)
-    stream = torch.cuda.Stream(device=dev)
-    for T in SWEEP_T:
-        s = pool.session_create_paused(T, T)
-        synth.fill_image_torch(pool.image(s), args.seed, s, L, HKV, D, T)
-        ms, ms_idle = [], []
-        for rep in range(12):
-            # even reps: device time (a spin keeps the stream busy while the host
-            # enqueues the resume, so the start event fires with its launches
-            # queued); odd reps: from an idle GPU, host enqueue included
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            if rep % 2 == 0:
-                with torch.cuda.stream(stream):
-                    torch.cuda._sleep(1_000_000)
-            a.record(stream)
-            pool.session_resume(s, stream)
-            b.record(stream)
-            torch.cuda.synchronize()
-            if rep >= 4:
-                (ms if rep % 2 == 0 else ms_idle).append(a.elapsed_time(b))
-            pool.session_pause(s, stream)
-        m = statistics.median(ms)
-        rw = 2 * T * TOKEN_BYTES / (m * 1e-3) / 1e9
-        resume.append({"T": T, "ms": round(m, 4), "gbs_rw": round(rw, 1), "frac": round(rw / peak, 3),
-                       "ms_from_idle_gpu": round(statistics.median(ms_idle), 4)})
-        pool.session_destroy(s)
-    pool.close()
     return {"decode": points, "resume": resume, "peak_gbs": peak}
 
 

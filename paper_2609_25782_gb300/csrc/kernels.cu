@@ -548,11 +548,12 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
 // Migration copy shape, from GB300 measurements of 2..16 loads per lane and
 // 4..16 CTAs per SM: 4 loads per lane over a grid of 16 CTAs per SM moves an
 // 8 x 32K-token burst at 0.97-0.98 of the copy bandwidth (0.93 with 8 x 8).
+constexpr int kMigChunkTokens = 16;     // tokens per migration item (divides bt)
 #ifndef KVT_MIG_UNROLL
 #define KVT_MIG_UNROLL 4          // 16-byte loads in flight per lane
 #endif
 #ifndef KVT_MIG_CTAS_PER_SM
-#define KVT_MIG_CTAS_PER_SM 16    // grid-stride CTAs of 256 threads per SM
+#define KVT_MIG_CTAS_PER_SM 32    // grid-stride CTAs of 256 threads per SM
 #endif
 
 __device__ __forceinline__ void st_out(uint4 *p, const uint4 &v) {
@@ -581,22 +582,25 @@ template <bool kPack>
 __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
     const Shape sh = a.s;
     const int runs = sh.L * 2 * sh.Hkv;
-    const int j0 = a.t_begin / sh.bt;
-    const int j1 = (a.t_end + sh.bt - 1) / sh.bt;
-    const int nj = j1 - j0;
-    const int items = runs * nj;
+    // Items are 16-token chunks of a run, so a 64-token block gives four
+    // warps the parallelism a 16-token block gives one.
+    const int q0 = a.t_begin / kMigChunkTokens;
+    const int q1 = (a.t_end + kMigChunkTokens - 1) / kMigChunkTokens;
+    const int nq = q1 - q0;
+    const int items = runs * nq;
     const int lane = threadIdx.x & 31;
     const int nwarps = (gridDim.x * blockDim.x) >> 5;
     for (int it = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; it < items; it += nwarps) {
-        const int c = it / nj;
-        const int j = j0 + (it - c * nj);
+        const int c = it / nq;
+        const int q = q0 + (it - c * nq);
+        const int j = q * kMigChunkTokens / sh.bt;
         const int blk = a.table[j];
         if (blk < 0 || blk >= sh.num_blocks) {
             if (lane == 0) atomicOr(a.err, kErrBadBlock);
             continue;
         }
-        const int t_lo = max(a.t_begin, j * sh.bt);
-        const int t_hi = min(a.t_end, (j + 1) * sh.bt);
+        const int t_lo = max(a.t_begin, q * kMigChunkTokens);
+        const int t_hi = min(a.t_end, (q + 1) * kMigChunkTokens);
         uint8_t *hp = a.hot + ((static_cast<int64_t>(blk) * runs + c) * sh.bt + (t_lo - j * sh.bt)) *
                                   kRowBytes;
         uint8_t *ip = a.img + (static_cast<int64_t>(c) * a.T_cap + t_lo) * kRowBytes;
@@ -817,15 +821,15 @@ static unsigned mig_grid(int64_t items, int num_sms, int max_ctas) {
 
 cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st) {
     if (a.t_end <= a.t_begin) return cudaSuccess;
-    const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
-    migrate_kernel<false><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
+    const int64_t nq = (a.t_end + kMigChunkTokens - 1) / kMigChunkTokens - a.t_begin / kMigChunkTokens;
+    migrate_kernel<false><<<mig_grid(nq * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_pack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st) {
     if (a.t_end <= a.t_begin) return cudaSuccess;
-    const int64_t nj = (a.t_end + a.s.bt - 1) / a.s.bt - a.t_begin / a.s.bt;
-    migrate_kernel<true><<<mig_grid(nj * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
+    const int64_t nq = (a.t_end + kMigChunkTokens - 1) / kMigChunkTokens - a.t_begin / kMigChunkTokens;
+    migrate_kernel<true><<<mig_grid(nq * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

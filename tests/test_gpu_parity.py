@@ -333,6 +333,42 @@ def test_round_trip_byte_identical(pkg, T):
     assert pool.check_device() == 0
 
 
+@pytest.mark.parametrize("bt,T1,T2", [(16, 37, 87), (64, 37, 87), (64, 64, 65), (64, 1, 300),
+                                       (64, 130, 1000)])
+def test_incremental_pack_resume_bit_exact(pkg, bt, T1, T2):
+    """Two pause/resume cycles: the second pack starts at the image's
+    watermark T1 (mid-block and mid-chunk for most cases), every resume
+    scatters into reshuffled blocks; images and blocks stay bit-exact."""
+    dev = torch.device("cuda:0")
+    L, NB, Hkv, D = 2, 80, 4, 128
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=NB, cold_bytes=1 << 26, max_sessions=2,
+                    max_batch=4, max_context=2048, alloc_seed=T2, block_tokens=bt)
+    s = pool.session_create(1024)
+    k, v = synth.kv_logical_torch(21, s, range(L), Hkv, D, 0, T2, dev)
+    kk, vv = k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+    pool.session_append(s, kk[:, :T1].contiguous(), vv[:, :T1].contiguous())
+    for cycle, T in enumerate((T1, T2)):
+        if cycle == 1:
+            pool.session_append(s, kk[:, T1:].contiguous(), vv[:, T1:].contiguous())
+        pool.session_pause(s)
+        torch.cuda.synchronize()
+        img = pool.image(s)
+        assert torch.equal(img[:, 0, :, :T].view(torch.int16), k[:, :, :T].view(torch.int16))
+        assert torch.equal(img[:, 1, :, :T].view(torch.int16), v[:, :, :T].view(torch.int16))
+        assert int(pool.session_info(s).cold_valid) == T
+        pool.shuffle_free(7 * T + cycle)
+        pool.session_resume(s)
+        row = pool.session_block_table(s)
+        assert len(row) == -(-T // bt)
+        blocks = pool.hot_view()[torch.as_tensor(row, device=dev, dtype=torch.int64)]
+        as_img = blocks.permute(1, 2, 3, 0, 4, 5).reshape(L, 2, Hkv, -1, D)[:, :, :, :T]
+        torch.cuda.synchronize()
+        assert torch.equal(as_img.view(torch.int16), img[:, :, :, :T].view(torch.int16))
+    assert pool.stats()["bytes_packed"] == T2 * pool.token_bytes     # each token written once
+    assert pool.check_device() == 0
+    pool.close()
+
+
 def test_config1_scenario(pkg):
     """Tiny single-layer case: 4 sessions (512..2048 tokens, one partial tail)
     decode; a 5th 1024-token session is packed, its blocks freed, the free
