@@ -509,9 +509,13 @@ def run_trace(args, rank, lru_factor: float = 0.0):
 
     from paper_2609_25782_gb300 import tiering_model
     sim_s = cfg.steps * cfg.dt_s
+    # mean KV a resident session holds, over all steps (every session stays resident)
+    mean_session = d.counts["session_tokens"] / (cfg.steps * cfg.sessions) * TOKEN_BYTES
     model = tiering_model.from_trace(
         cold_write_bytes=st["bytes_packed"], hot_read_bytes=d.counts["decode_tokens"] * TOKEN_BYTES,
-        cold_read_bytes=st["bytes_unpacked"], simulated_seconds=sim_s)
+        cold_read_bytes=st["bytes_unpacked"], simulated_seconds=sim_s,
+        mean_session_bytes=mean_session,
+        hbm_bytes=torch.cuda.get_device_properties(dev).total_memory)
     extra = {"model": {k: (round(v, 3) if isinstance(v, float) and v != float("inf") else
                            (None if v == float("inf") else v)) for k, v in model.items()},
              "simulated_s": sim_s}

@@ -7,6 +7,9 @@
 * Read power (Section 4, "Methodology"): the sum over memory tiers of each
   tier's read rate times its energy per bit. Serving the hot set from flash
   instead of HBM costs (E_flash - E_HBM) * (hot-set read rate) more.
+* Session capacity (Section 4, "Capacity and latency"): the memory left for
+  KV (HBM minus the resident weights, plus the cold tier when there is one)
+  divided by the mean KV a resident session holds.
 
 The counters come from a trace run: bytes written to the cold tier by pauses
 and evictions, bytes decode read from the hot set, and the simulated time the
@@ -15,6 +18,7 @@ trace covers (steps x seconds per step).
 from __future__ import annotations
 
 SECONDS_PER_YEAR = 365.25 * 24 * 3600
+GIB = 1024 ** 3
 TIB = 1024 ** 4
 
 # Parameters the paper uses for its modelled HBF tier (Section 4).
@@ -22,6 +26,8 @@ HBF_CAPACITY_BYTES = 3 * TIB
 HBF_PE_CYCLES = 100_000
 HBF_WAF = 1.02
 HBM_PJ_PER_BIT = 3.5
+WEIGHT_BYTES = 56.8 * GIB          # Qwen3-Coder-30B-A3B bf16 weights, kept in HBM (Section 4)
+PAPER_HBM_BYTES = 192 * GIB        # the modelled node's HBM (Section 4)
 
 
 def lifetime_seconds(write_rate_bytes_per_s: float, capacity_bytes: float = HBF_CAPACITY_BYTES,
@@ -48,9 +54,19 @@ def hot_set_power_gap_watts(hot_read_rate_bytes_per_s: float, flash_pj_per_bit: 
         read_power_watts({"hbm": hot_read_rate_bytes_per_s}, {"hbm": hbm_pj_per_bit})
 
 
+def session_capacity(mean_session_bytes: float, hbm_bytes: float,
+                     weight_bytes: float = WEIGHT_BYTES, cold_tier_bytes: float = 0.0) -> float:
+    """Concurrent sessions whose KV fits in HBM (and the cold tier, if any)
+    next to the weights, at a mean resident footprint per session."""
+    return (hbm_bytes - weight_bytes + cold_tier_bytes) / mean_session_bytes
+
+
 def from_trace(cold_write_bytes: float, hot_read_bytes: float, cold_read_bytes: float,
-               simulated_seconds: float, flash_pj_per_bit: float = 20.0) -> dict:
-    """Lifetime and read power of one GPU under a measured trace."""
+               simulated_seconds: float, flash_pj_per_bit: float = 20.0,
+               mean_session_bytes: float | None = None, hbm_bytes: float | None = None) -> dict:
+    """Lifetime and read power of one GPU under a measured trace; with the
+    trace's mean resident KV per session and the GPU's HBM size, also the
+    sessions that fit with HBM alone and with the cold tier added."""
     rw = cold_write_bytes / simulated_seconds
     hot = hot_read_bytes / simulated_seconds
     cold = cold_read_bytes / simulated_seconds
@@ -64,4 +80,9 @@ def from_trace(cold_write_bytes: float, hot_read_bytes: float, cold_read_bytes: 
         "read_power_w_all_from_flash": read_power_watts({"flash": hot + cold},
                                                         {"flash": flash_pj_per_bit}),
         "flash_pj_per_bit": flash_pj_per_bit,
-    }
+    } | ({} if mean_session_bytes is None or hbm_bytes is None else {
+        "mean_session_gib": mean_session_bytes / GIB,
+        "sessions_hbm_only": session_capacity(mean_session_bytes, hbm_bytes),
+        "sessions_with_cold_tier": session_capacity(mean_session_bytes, hbm_bytes,
+                                                    cold_tier_bytes=HBF_CAPACITY_BYTES),
+    })

@@ -113,7 +113,8 @@ class TraceDriver:
         self.peak_tokens = list(self.tokens)
         self.peak_blocks = 0
         self.counts = {"resumes": 0, "pauses": 0, "appended_tokens": 0, "decode_tokens": 0,
-                       "turn_tokens": 0, "steps": 0}
+                       "turn_tokens": 0, "steps": 0,
+                       "session_tokens": 0}   # sum over steps of all sessions' lengths
         self.step_events = []                # (start, end) per step (gpu)
         self.mig_events = []                 # (kind, start, end, bytes)
         self.admit_ev = {}
@@ -269,6 +270,7 @@ class TraceDriver:
                 if self.burst_left[i] <= 0:
                     self.retire.append(i)
         self.counts["steps"] += 1
+        self.counts["session_tokens"] += sum(self.tokens)
 
     def run(self, steps: int | None = None) -> None:
         for k in range(self.cfg.steps if steps is None else steps):

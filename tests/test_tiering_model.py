@@ -3,7 +3,10 @@
 Pinned to figures the paper prints: its 950 W per device at 20 pJ/bit and
 its 2.1 / 7.6 / 12.2 kW per 8-GPU node at 8 / 20 / 30 pJ/bit must all follow
 from one hot-set read rate under the same power model (Section 4, "Read
-energy"); no write means unbounded lifetime (Section 4, "Endurance").
+energy"); no write means unbounded lifetime (Section 4, "Endurance"); its
+165 sessions for HBM alone, 3,900 with a 3 TiB cold tier and the 24x ratio
+must follow from its 0.82 GiB mean footprint (Section 4, "Capacity and
+latency").
 """
 import math
 
@@ -44,3 +47,25 @@ def test_from_trace(tm):
     tiered = 1e10 * 8 * 3.5e-12 + 1e8 * 8 * 20e-12
     assert r["read_power_w_tiered"] == pytest.approx(tiered)
     assert r["read_power_w_all_from_flash"] > r["read_power_w_tiered"]
+
+
+def test_paper_capacity_figures(tm):
+    mean = 0.82 * tm.GIB                       # resident KV per session, steady state
+    hbm_only = tm.session_capacity(mean, tm.PAPER_HBM_BYTES)
+    tiered = tm.session_capacity(mean, tm.PAPER_HBM_BYTES, cold_tier_bytes=tm.HBF_CAPACITY_BYTES)
+    assert abs(hbm_only - 165) < 1.0           # "saturates at 165 sessions"
+    assert abs(tiered / 3900 - 1) < 0.01       # "expands capacity to 3,900 sessions"
+    assert round(tiered / hbm_only) == 24      # "24x more concurrent sessions"
+    # the cold tier adds to what HBM holds; without the weights' share both would be off
+    assert abs(tm.HBF_CAPACITY_BYTES / mean / 3900 - 1) > 0.03
+    assert tm.session_capacity(mean, tm.PAPER_HBM_BYTES, weight_bytes=0) > 230
+
+
+def test_from_trace_capacity(tm):
+    r = tm.from_trace(cold_write_bytes=0, hot_read_bytes=1e12, cold_read_bytes=0,
+                      simulated_seconds=1.0, mean_session_bytes=1.0 * tm.GIB,
+                      hbm_bytes=tm.PAPER_HBM_BYTES)
+    assert r["mean_session_gib"] == pytest.approx(1.0)
+    assert r["sessions_hbm_only"] == pytest.approx(192 - 56.8)
+    assert r["sessions_with_cold_tier"] == pytest.approx(192 - 56.8 + 3072)
+    assert "sessions_hbm_only" not in tm.from_trace(0, 1, 0, 1.0)
