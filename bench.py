@@ -548,6 +548,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
         "decode_kv_gb": round(d.counts["decode_tokens"] * TOKEN_BYTES / 1e9, 1),
         "hot_read_share": round(d.counts["decode_tokens"] * TOKEN_BYTES /
                                 (d.counts["decode_tokens"] * TOKEN_BYTES + mig["unpack"][1]), 4),
+        # the hot set's share of resident KV (the paper's counterpart of the read share)
+        "hot_set_capacity_share": round(d.counts["decode_tokens"] / d.counts["session_tokens"], 4),
         "device_flags": flags,
         "trace": "seeded synthetic: T0 U[2K,24K], bursts Geometric(200), pauses Exp(30 s), "
                  "turn append LogNormal(median 1536, sigma 1, cap 16K), dt 75 ms/step",
