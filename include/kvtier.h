@@ -167,7 +167,7 @@ int session_create_paused(kv_pool *pool, int64_t max_tokens, int64_t tokens,
 int session_destroy(kv_pool *pool, int32_t sid);
 
 /* Data path 3 (Section 3): write n >= 1 new tokens of an ACTIVE session.
- * k, v: device, bf16 [L][n][Hkv][D] contiguous. Blocks are popped from the
+ * k, v: device, bf16 [L][n][Hkv][D] contiguous, 16-byte aligned. Blocks are popped from the
  * free list when the tail block fills; tokens go to positions T .. T+n-1,
  * then T += n. The stream first waits for the session's last resume.
  * Errors: KV_ERR_BAD_STATE (paused), KV_ERR_NO_HOT_BLOCKS, capacity
@@ -184,7 +184,9 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  *                blocks in logical order
  *   seq_lens     device int32 [B]; 1 <= seq_lens[b] <= max_blocks * bt
  *   scale        multiplies q.k before the softmax (1/sqrt(D) usually)
- *   out          device fp32 [B][Hq][D]   (or [L][B][Hq][D])
+ *   out          device fp32 [B][Hq][D]   (or [L][B][Hq][D]), 16-byte aligned
+ *                (q, block_tables and seq_lens 4-byte aligned; misaligned
+ *                pointers -> KV_ERR_INVALID_ARG)
  * out[b][h] = sum_i softmax_i(scale * q[b][h] . K[g][i]) V[g][i] over the
  * session's tokens i < seq_lens[b], g = h / (Hq/Hkv). Tokens past seq_len
  * in the last block are never read into the result (they may hold NaN).

@@ -63,6 +63,11 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
                                         kv_stream_t stream) {
     if (!cfg || !q || !block_tables || !seq_lens || !out || !cfg->hot_base)
         return fail(KV_ERR_INVALID_ARG, "decode_attention_noalloc: null pointer");
+    if (((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(block_tables) |
+          reinterpret_cast<uintptr_t>(seq_lens)) & 3) || (reinterpret_cast<uintptr_t>(out) & 15))
+        return fail(KV_ERR_INVALID_ARG,
+                    "decode_attention_noalloc: q, block_tables, seq_lens need 4-byte and out "
+                    "16-byte alignment");
     const kv_pool_config &c = *cfg;
     const int G = c.num_kv_heads > 0 ? c.num_q_heads / c.num_kv_heads : 0;
     if (c.head_dim != kvt::kHeadDim || (c.block_tokens != 16 && c.block_tokens != 64) ||

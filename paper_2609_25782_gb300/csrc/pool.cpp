@@ -525,6 +525,14 @@ int session_destroy(kv_pool *p, int32_t sid) {
     return KV_OK;
 }
 
+// The decode kernels read q as 4-byte words and store out as 16-byte vectors.
+static bool decode_pointers_aligned(const void *q, const void *tables, const void *lens,
+                                    const void *out) {
+    const uintptr_t a4 = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(tables) |
+                         reinterpret_cast<uintptr_t>(lens);
+    return (a4 & 3) == 0 && (reinterpret_cast<uintptr_t>(out) & 15) == 0;
+}
+
 static int ensure_event(kv_pool *p, cudaEvent_t *ev) {
     if (*ev || p->host_only) return KV_OK;
     return p->cuda("cudaEventCreate",
@@ -545,6 +553,8 @@ static int lru_append(kv_pool *p, int32_t sid, const void *k, const void *v, int
     if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "append to a paused session");
     if (n < 1) return fail(KV_ERR_INVALID_ARG, "n must be >= 1");
     if (!p->host_only && (!k || !v)) return fail(KV_ERR_INVALID_ARG, "null k or v");
+    if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
+        return fail(KV_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
     if (s->T + n > s->cap) return fail(KV_ERR_INVALID_ARG, "append past the session capacity");
     const int bt = p->cfg.block_tokens;
     const int64_t have = static_cast<int64_t>(s->blocks.size());
@@ -721,6 +731,8 @@ int session_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_
     if (s->state != KV_SESSION_ACTIVE) return fail(KV_ERR_BAD_STATE, "append to a paused session");
     if (n < 1) return fail(KV_ERR_INVALID_ARG, "n must be >= 1");
     if (!p->host_only && (!k || !v)) return fail(KV_ERR_INVALID_ARG, "null k or v");
+    if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) & 15)
+        return fail(KV_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
     if (s->T + n > s->cap) return fail(KV_ERR_INVALID_ARG, "append past the session capacity");
     const int bt = p->cfg.block_tokens;
     const int64_t have = static_cast<int64_t>(s->blocks.size());
@@ -779,8 +791,10 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
     if (flags & ~static_cast<uint32_t>(KV_DECODE_OVERLAP_PREVIOUS | KV_DECODE_OUT_BF16))
         return fail(KV_ERR_INVALID_ARG, "unknown decode flag");
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
-    if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
     if (!q || !block_tables || !seq_lens || !out) return fail(KV_ERR_INVALID_ARG, "null pointer");
+    if (!decode_pointers_aligned(q, block_tables, seq_lens, out))
+        return fail(KV_ERR_INVALID_ARG, "q, block_tables, seq_lens need 4-byte and out 16-byte alignment");
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
     if (layer < -1 || layer >= p->cfg.num_layers) return fail(KV_ERR_INVALID_ARG, "bad layer");
     const int nl = layer < 0 ? p->cfg.num_layers : 1;
     if (B < 1 || static_cast<int64_t>(nl) * B > 65535)

@@ -39,7 +39,10 @@ int main(void) {
     kv_pool_stats st;
     int32_t s0 = -1, s1 = -1;
     int32_t batch[2];
-    float out_dummy = 0.0f;
+    float scratch[8];
+    /* a 16-byte-aligned stand-in for the device buffers (never dereferenced on
+       a host-logic pool) */
+    float *out_dummy = (float *)(((uintptr_t)scratch + 15) & ~(uintptr_t)15);
 
     memset(&cfg, 0, sizeof cfg);
     cfg.num_layers = 48;
@@ -88,8 +91,11 @@ int main(void) {
     expect_code("resume active", session_resume(pool, s0, NULL), KV_ERR_BAD_STATE);
     printf("last_error_nonempty=%d\n", kv_last_error()[0] != '\0');
     expect_code("decode on host-logic pool",
-                decode_attention(pool, 0, &out_dummy, batch, batch, 1, 1, 1.0f, &out_dummy, NULL),
+                decode_attention(pool, 0, out_dummy, batch, batch, 1, 1, 1.0f, out_dummy, NULL),
                 KV_ERR_BAD_STATE);
+    expect_code("decode with misaligned out",
+                decode_attention(pool, 0, out_dummy, batch, batch, 1, 1, 1.0f, out_dummy + 1, NULL),
+                KV_ERR_INVALID_ARG);
     expect_code("append past capacity", session_append(pool, s1, NULL, NULL, 500, NULL),
                 KV_ERR_INVALID_ARG);
     batch[1] = s0;

@@ -108,7 +108,8 @@ def test_random_calls_keep_invariants(kv, lru, seed):
 
 
 def test_decode_flags_and_arguments_rejected(kv):
-    cfg = kv.make_config(num_layers=2, num_hot_blocks=8, flags=kv.KV_POOL_HOST_LOGIC_ONLY)
+    cfg = kv.make_config(num_layers=2, num_hot_blocks=8, flags=kv.KV_POOL_HOST_LOGIC_ONLY,
+                         cold_bytes=1 << 24)
     pool = kv.kv_pool_create(cfg)
     with pytest.raises(kv.KVError) as e:
         kv.decode_attention_ex(pool, 0, 1, 1, 1, 1, 1, 1.0, 1, 1 << 7, None)
@@ -122,11 +123,24 @@ def test_decode_flags_and_arguments_rejected(kv):
         with pytest.raises(kv.KVError) as e:
             kv.decode_append_attention(pool, 0, 1024, kn, vn, 2048, 4096, 1, 1, 1.0, 8192)
         assert e.value.code == code
+    for args in ((1026, 2048, 4096, 8192), (1024, 2048, 4096, 8200), (1024, 2050, 4096, 8192)):
+        with pytest.raises(kv.KVError) as e:       # misaligned q, out, block_tables
+            kv.decode_attention(pool, 0, args[0], args[1], args[2], 1, 1, 1.0, args[3], None)
+        assert e.value.code == kv.KV_ERR_INVALID_ARG and "align" in kv.kv_last_error()
+    sid = kv.session_create(pool, 64)
+    with pytest.raises(kv.KVError) as e:
+        kv.session_append(pool, sid, 1032, 1024, 1, None)
+    assert e.value.code == kv.KV_ERR_INVALID_ARG
+    kv.session_append(pool, sid, 1024, 2048, 1, None)   # aligned: accepted (host logic only)
     kv.kv_pool_inject_decode_timeout(pool, 1)          # armed, then disarmed: host state only
     kv.kv_pool_inject_decode_timeout(pool, 0)
     kv.kv_pool_destroy(pool)
     with pytest.raises(kv.KVError) as e:
         kv.kv_pool_inject_decode_timeout(None, 1)
+    assert e.value.code == kv.KV_ERR_INVALID_ARG
+    with pytest.raises(kv.KVError) as e:              # no-alloc path: misaligned out
+        kv.decode_attention_noalloc(kv.make_config(num_layers=2, num_hot_blocks=8, hot_base=256),
+                                    0, 1024, 2048, 4096, 1, 1, 1.0, 8200)
     assert e.value.code == kv.KV_ERR_INVALID_ARG
     with pytest.raises(kv.KVError) as e:              # no-alloc path: bad shapes, before any CUDA call
         kv.decode_attention_noalloc(kv.make_config(num_layers=2, num_hot_blocks=8, head_dim=64,

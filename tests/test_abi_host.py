@@ -101,7 +101,7 @@ def test_state_machine_errors(kv):
             fn()
         assert e.value.code == kv.KV_ERR_BAD_STATE
     with pytest.raises(kv.KVError) as e:
-        kv.decode_attention(pool, 0, 1, 1, 1, 1, 1, 1.0, 1, None)
+        kv.decode_attention(pool, 0, 256, 512, 768, 1, 1, 1.0, 1024, None)   # aligned dummies
     assert e.value.code == kv.KV_ERR_BAD_STATE
     with pytest.raises(kv.KVError) as e:
         kv.session_info(pool, 5)
