@@ -1010,6 +1010,8 @@ int kv_pool_batch_tables(kv_pool *p, const int32_t *sids, int32_t B, int32_t *bl
     if (p->host_only && !p->lru)
         return fail(KV_ERR_BAD_STATE, "batch tables on a host-logic-only pool");
     if (!p->host_only && (!block_tables || !seq_lens)) return fail(KV_ERR_INVALID_ARG, "null output");
+    if ((reinterpret_cast<uintptr_t>(block_tables) | reinterpret_cast<uintptr_t>(seq_lens)) & 3)
+        return fail(KV_ERR_INVALID_ARG, "block_tables and seq_lens must be 4-byte aligned");
     if (max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "max_blocks must be >= 1");
     for (int32_t i = 0; i < B; ++i) {
         Session *s = p->session(sids[i]);
@@ -1037,6 +1039,8 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
                           int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream_) {
     if (!p || !sids || B < 1) return fail(KV_ERR_INVALID_ARG, "bad argument");
     if (!p->host_only && (!block_tables || !seq_lens)) return fail(KV_ERR_INVALID_ARG, "null output");
+    if ((reinterpret_cast<uintptr_t>(block_tables) | reinterpret_cast<uintptr_t>(seq_lens)) & 3)
+        return fail(KV_ERR_INVALID_ARG, "block_tables and seq_lens must be 4-byte aligned");
     if (max_blocks < 1) return fail(KV_ERR_INVALID_ARG, "max_blocks must be >= 1");
     const int bt = p->cfg.block_tokens;
     const std::vector<int32_t> members(sids, sids + B);

@@ -132,6 +132,9 @@ def test_decode_flags_and_arguments_rejected(kv):
         kv.session_append(pool, sid, 1032, 1024, 1, None)
     assert e.value.code == kv.KV_ERR_INVALID_ARG
     kv.session_append(pool, sid, 1024, 2048, 1, None)   # aligned: accepted (host logic only)
+    with pytest.raises(kv.KVError) as e:               # misaligned batch outputs
+        kv.kv_pool_batch_reserve(pool, [sid], 1026, 4, 2048, None)
+    assert e.value.code == kv.KV_ERR_INVALID_ARG
     kv.kv_pool_inject_decode_timeout(pool, 1)          # armed, then disarmed: host state only
     kv.kv_pool_inject_decode_timeout(pool, 0)
     kv.kv_pool_destroy(pool)
