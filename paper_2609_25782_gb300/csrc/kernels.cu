@@ -629,23 +629,29 @@ template <bool kPack>
 __global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__ BlockJobs a) {
     const Shape sh = a.s;
     const int runs = sh.L * 2 * sh.Hkv;
-    const int items = a.n * runs;
+    const int cpb = sh.bt / kMigChunkTokens;      // 16-token chunks per block
+    const int items = a.n * runs * cpb;
     const int lane = threadIdx.x & 31;
     const int nwarps = (gridDim.x * blockDim.x) >> 5;
     for (int it = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; it < items; it += nwarps) {
-        const int jb = it / runs;
-        const int c = it - jb * runs;
+        const int jb = it / (runs * cpb);
+        const int rem = it - jb * runs * cpb;
+        const int c = rem / cpb;
+        const int ch = rem - c * cpb;
         const BlockJob &b = a.job[jb];
         if (b.slot < 0 || b.slot >= sh.num_blocks || b.t0 < 0 || b.t1 > sh.bt) {
-            if (lane == 0) atomicOr(a.err, kErrBadBlock);
+            if (lane == 0 && ch == 0 && c == 0) atomicOr(a.err, kErrBadBlock);
             continue;
         }
-        uint8_t *hp = a.hot + ((static_cast<int64_t>(b.slot) * runs + c) * sh.bt + b.t0) * kRowBytes;
+        const int t_lo = max(b.t0, ch * kMigChunkTokens);
+        const int t_hi = min(b.t1, (ch + 1) * kMigChunkTokens);
+        if (t_hi <= t_lo) continue;
+        uint8_t *hp = a.hot + ((static_cast<int64_t>(b.slot) * runs + c) * sh.bt + t_lo) * kRowBytes;
         uint8_t *ip = b.img + (static_cast<int64_t>(c) * b.T_cap + static_cast<int64_t>(b.j) * sh.bt +
-                               b.t0) * kRowBytes;
+                               t_lo) * kRowBytes;
         const uint4 *src = reinterpret_cast<const uint4 *>(kPack ? hp : ip);
         uint4 *dst = reinterpret_cast<uint4 *>(kPack ? ip : hp);
-        const int units = (b.t1 - b.t0) * (kRowBytes / 16);
+        const int units = (t_hi - t_lo) * (kRowBytes / 16);
         for (int u0 = 0; u0 < units; u0 += 32 * KVT_MIG_UNROLL) {
             uint4 v[KVT_MIG_UNROLL];
 #pragma unroll
@@ -845,8 +851,8 @@ cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st) {
 cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, int max_ctas,
                               cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    const unsigned grid =
-        mig_grid(static_cast<int64_t>(a.n) * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas);
+    const unsigned grid = mig_grid(static_cast<int64_t>(a.n) * a.s.L * 2 * a.s.Hkv *
+                                       (a.s.bt / kMigChunkTokens), num_sms, max_ctas);
     if (pack)
         block_jobs_kernel<true><<<grid, 256, 0, st>>>(a);
     else

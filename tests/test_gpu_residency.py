@@ -26,19 +26,21 @@ def bits(t):
     return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
 
 
-@pytest.mark.parametrize("fused", [False, True])
-def test_residency_random_sequence(cuda_dev, fused):
+@pytest.mark.parametrize("fused,bt", [(False, 16), (True, 16), (True, 64)])
+def test_residency_random_sequence(cuda_dev, fused, bt):
     """fused: decode batches take their step token with the decode
-    (kv_pool_batch_reserve + decode_append_attention, all layers)."""
+    (kv_pool_batch_reserve + decode_append_attention, all layers). bt 64:
+    evictions and fetches move 64-token blocks as four 16-token chunks."""
     import __graft_entry__
     __graft_entry__.build()
     from paper_2609_25782_gb300 import Pool, kvtier
 
-    L, Hq, Hkv, D, bt, nb, seed = 2, 32, 4, 128, 16, 40, 8
+    L, Hq, Hkv, D, seed = 2, 32, 4, 128, 8
+    nb = 40 if bt == 16 else 16                     # about the same pressure in tokens
     cap = 600
     pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=10 * cap * pool_token_bytes(L, Hkv),
                 max_sessions=10, max_batch=L * 4, max_context=cap, alloc_seed=seed,
-                lru_residency=True)
+                lru_residency=True, block_tokens=bt)
     o = ResidencyOracle(nb, bt, seed=seed, token_bytes=pool.token_bytes)
     rnd = random.Random(seed)
     st = torch.cuda.Stream()
