@@ -181,7 +181,9 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  *                then carry a leading [L] dimension)
  *   q            device bf16 [B][Hq][D]   (or [L][B][Hq][D])
  *   block_tables device int32 [B][max_blocks]; row b lists session b's
- *                blocks in logical order
+ *                blocks in logical order. max_blocks sizes the grid (splits
+ *                for max_blocks * bt tokens): the batch's longest session is
+ *                the best width
  *   seq_lens     device int32 [B]; 1 <= seq_lens[b] <= max_blocks * bt
  *   scale        multiplies q.k before the softmax (1/sqrt(D) usually)
  *   out          device fp32 [B][Hq][D]   (or [L][B][Hq][D]), 16-byte aligned

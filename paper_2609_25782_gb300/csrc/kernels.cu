@@ -43,6 +43,9 @@ constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
 // per SM; smaller grids get deeper rings so each SM still keeps ~24 tiles
 // in flight. The depth changes only the prefetch distance, never which warp
 // takes which tile, so all variants give bit-identical results.
+#ifndef KVT_WAVE_MARGIN
+#define KVT_WAVE_MARGIN 0.1   // last-wave fill gain that moves a grid to 2 CTAs per SM
+#endif
 constexpr int kStagesFull = KVT_STAGES;    // 3 CTAs per SM
 constexpr int kStagesHalf = 3;             // 2 CTAs per SM
 constexpr int kStagesOne = 6;              // 1 CTA per SM
@@ -789,11 +792,17 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
     // CTAs of the grid (an upper bound: splits past a session's own count
     // exit at once) against the SMs decide the ring depth.
     const int64_t ctas = static_cast<int64_t>(splits) * a.s.Hkv * a.nlayers * a.B;
+    // Beyond two CTAs per SM, 2 per SM still wins when it fills its last wave
+    // clearly better than 3 per SM (a grid just above one 3-per-SM wave).
+    auto fill = [&](int per_sm) {
+        const double w = static_cast<double>(ctas) / (per_sm * static_cast<double>(num_sms));
+        return w / static_cast<double>(static_cast<int64_t>(w) + (w > static_cast<int64_t>(w)));
+    };
     cudaError_t e;
     if (ctas <= num_sms) {
         c1.dynamicSmemBytes = decode_smem(kStagesOne);
         e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesOne>, map, a);
-    } else if (ctas <= 2 * static_cast<int64_t>(num_sms)) {
+    } else if (ctas <= 2 * static_cast<int64_t>(num_sms) || fill(2) > fill(3) + KVT_WAVE_MARGIN) {
         c1.dynamicSmemBytes = decode_smem(kStagesHalf);
         e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesHalf>, map, a);
     } else {

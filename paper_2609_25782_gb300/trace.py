@@ -221,11 +221,14 @@ class TraceDriver:
                         self.dstream.wait_event(ev)
             sids = [self.sids[i] for i in members]
             B = len(sids)
+            # tables as wide as this batch's longest session (after its step token):
+            # no launched split lies past every session's end
+            mb = -(-(max(self.tokens[i] for i in members) + 1) // cfg.block_tokens)
             if cfg.fused_append:             # this step's token (path 3) comes with the decode
                 if self.gpu:
                     with self._torch.cuda.stream(self.dstream):
                         k_new, v_new = self._step_kv(members)
-                    kvtier.kv_pool_batch_reserve(self.pool, sids, self.tables, self.max_blocks,
+                    kvtier.kv_pool_batch_reserve(self.pool, sids, self.tables, mb,
                                                  self.seq_lens, self.dstream)
                 else:
                     kvtier.kv_pool_batch_reserve(self.pool, sids, None, 1 << 20, None, None)
@@ -238,7 +241,7 @@ class TraceDriver:
                 if not self.gpu and cfg.lru:     # recency and spilled-block fetches
                     kvtier.kv_pool_batch_tables(self.pool, sids, None, 1 << 20, None, None)
                 if self.gpu:
-                    kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, self.max_blocks,
+                    kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, mb,
                                                 self.seq_lens, self.dstream)
             self.counts["appended_tokens"] += len(members)
             blocks = sum(-(-self.tokens[i] // cfg.block_tokens)
@@ -252,12 +255,12 @@ class TraceDriver:
                     if cfg.fused_append:
                         kvtier.decode_append_attention(
                             self.pool, l, self.q[l], k_new[l], v_new[l], self.tables,
-                            self.seq_lens, B, self.max_blocks, 1 / math.sqrt(128), self.out[l],
+                            self.seq_lens, B, mb, 1 / math.sqrt(128), self.out[l],
                             flags, self.dstream)
                     else:
                         kvtier.decode_attention_ex(
                             self.pool, l, self.q[l], self.tables, self.seq_lens, B,
-                            self.max_blocks, 1 / math.sqrt(128), self.out[l], flags,
+                            mb, 1 / math.sqrt(128), self.out[l], flags,
                             self.dstream)
                 end.record(self.dstream)
                 self.last_decode_ev = end
