@@ -581,8 +581,9 @@ __device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
 // Both sides of a run are contiguous rows of 256 B; a warp moves it with
 // 16-byte loads, KVT_MIG_UNROLL in flight per lane. Items are ordered run-major so
 // that consecutive warps walk the image sequentially.
-template <bool kPack>
-__global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
+// The copy loop of a session's migration; block_of(j) gives logical block j's slot.
+template <bool kPack, typename BlockOf>
+__device__ __forceinline__ void migrate_runs(const MigArgs &a, BlockOf block_of) {
     const Shape sh = a.s;
     const int runs = sh.L * 2 * sh.Hkv;
     // Items are 16-token chunks of a run, so a 64-token block gives four
@@ -597,7 +598,7 @@ __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
         const int c = it / nq;
         const int q = q0 + (it - c * nq);
         const int j = q * kMigChunkTokens / sh.bt;
-        const int blk = a.table[j];
+        const int blk = block_of(j);
         if (blk < 0 || blk >= sh.num_blocks) {
             if (lane == 0) atomicOr(a.err, kErrBadBlock);
             continue;
@@ -628,6 +629,21 @@ __global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
 
 // K3'/K4': block-granular moves for the residency mode: one warp per
 // (job, layer, K|V, kv-head) run; a job moves tokens [t0, t1) of one block.
+template <bool kPack>
+__global__ void __launch_bounds__(256) migrate_kernel(const MigArgs a) {
+    migrate_runs<kPack>(a, [&](int j) { return a.table[j]; });
+}
+
+// Resume-unpack with the new block ids in the launch parameters: the grid
+// also writes them to the session's table row (read by later work only).
+__global__ void __launch_bounds__(256) resume_inline_kernel(const __grid_constant__ ResumeArgs r) {
+    const int nthreads = gridDim.x * blockDim.x;
+    int32_t *row = const_cast<int32_t *>(r.m.table);   // the pool's own row: writable
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < r.n; j += nthreads)
+        row[j] = r.blocks[j];
+    migrate_runs<false>(r.m, [&](int j) { return j < r.n ? r.blocks[j] : -1; });
+}
+
 template <bool kPack>
 __global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__ BlockJobs a) {
     const Shape sh = a.s;
@@ -838,6 +854,14 @@ cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStrea
     if (a.t_end <= a.t_begin) return cudaSuccess;
     const int64_t nq = (a.t_end + kMigChunkTokens - 1) / kMigChunkTokens - a.t_begin / kMigChunkTokens;
     migrate_kernel<false><<<mig_grid(nq * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_unpack_inline(const ResumeArgs &r, int num_sms, int max_ctas, cudaStream_t st) {
+    const MigArgs &a = r.m;
+    if (a.t_end <= a.t_begin || r.n < 1 || r.n > kResumeInlineMax) return cudaErrorInvalidValue;
+    const int64_t nq = (a.t_end + kMigChunkTokens - 1) / kMigChunkTokens - a.t_begin / kMigChunkTokens;
+    resume_inline_kernel<<<mig_grid(nq * a.s.L * 2 * a.s.Hkv, num_sms, max_ctas), 256, 0, st>>>(r);
     return cudaGetLastError();
 }
 

@@ -88,6 +88,16 @@ struct MigArgs {
     Shape s;
 };
 
+// A resume whose new block ids ride in the launch: the kernel writes the
+// session's table row itself and needs no prior table-write launch.
+constexpr int kResumeInlineMax = 2048;   // blocks (32K tokens at bt = 16)
+struct ResumeArgs {
+    MigArgs m;                // m.table: the session's device row, written here
+    int32_t n;                // blocks in the row
+    int32_t pad;
+    int32_t blocks[kResumeInlineMax];
+};
+
 struct AppendArgs {
     const uint8_t *k, *v;     // [L][n][Hkv][D] bf16
     const int32_t *table;
@@ -146,6 +156,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
                           cudaStream_t st, bool overlap_previous);
 // max_ctas > 0 caps the migration grids (kv_pool_set_migration_limit).
 cudaError_t launch_unpack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);
+cudaError_t launch_unpack_inline(const ResumeArgs &r, int num_sms, int max_ctas, cudaStream_t st);
 cudaError_t launch_pack(const MigArgs &a, int num_sms, int max_ctas, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_block_jobs(const BlockJobs &a, bool pack, int num_sms, int max_ctas,

@@ -60,6 +60,8 @@ struct Session {
     bool ready_recorded = false;
     cudaEvent_t appended = nullptr;
     bool appended_recorded = false;
+    int16_t pack_fence = -1;          // simple mode: fence slot and generation of the
+    uint64_t pack_gen = 0;            // last pause's pack (it reads the table row)
 };
 
 // A planned eviction: block j of session sid leaves hot slot `slot`; tokens
@@ -892,6 +894,8 @@ int session_pause(kv_pool *p, int32_t sid, kv_stream_t stream_) {
     p->next_fence = (f + 1) % kFenceSlots;
     const uint64_t gen = ++p->fence_gen;
     p->fences[f].gen = gen;
+    s->pack_fence = static_cast<int16_t>(f);
+    s->pack_gen = gen;
     for (int32_t b : s->blocks) {
         p->free_list.push_back(b);
         p->block_fence[b] = static_cast<int16_t>(f);
@@ -926,12 +930,32 @@ int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
 
     int rc = ensure_event(p, &s->ready);
     if (!rc) rc = p->wait_fences(fresh.data(), fresh.size(), st);
-    if (!rc) rc = p->write_table(sid, fresh.data(), 0, need, st);
-    if (!rc) {
-        kvt::MigArgs m = p->mig_args(sid, *s);
-        m.t_begin = 0;
-        m.t_end = static_cast<int32_t>(s->T);
-        rc = p->cuda("unpack launch", [&] { return kvt::launch_unpack(m, p->num_sms, p->mig_ctas, st); });
+    // The session's own last pack reads the table row this resume rewrites:
+    // order after it while its fence slot still holds that pack (a re-recorded
+    // slot means it was synchronised first).
+    if (!rc && s->pack_fence >= 0 && p->fences[s->pack_fence].gen == s->pack_gen)
+        rc = p->cuda("cudaStreamWaitEvent",
+                     [&] { return cudaStreamWaitEvent(st, p->fences[s->pack_fence].ev, 0); });
+    if (!rc && need <= kvt::kResumeInlineMax) {
+        // one launch: the block ids ride in the parameters, the kernel writes the row
+        kvt::ResumeArgs r;
+        r.m = p->mig_args(sid, *s);
+        r.m.t_begin = 0;
+        r.m.t_end = static_cast<int32_t>(s->T);
+        r.n = static_cast<int32_t>(need);
+        r.pad = 0;
+        std::memcpy(r.blocks, fresh.data(), sizeof(int32_t) * need);
+        rc = p->cuda("unpack launch",
+                     [&] { return kvt::launch_unpack_inline(r, p->num_sms, p->mig_ctas, st); });
+    } else if (!rc) {
+        rc = p->write_table(sid, fresh.data(), 0, need, st);
+        if (!rc) {
+            kvt::MigArgs m = p->mig_args(sid, *s);
+            m.t_begin = 0;
+            m.t_end = static_cast<int32_t>(s->T);
+            rc = p->cuda("unpack launch",
+                         [&] { return kvt::launch_unpack(m, p->num_sms, p->mig_ctas, st); });
+        }
     }
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
     if (rc) return rc;
