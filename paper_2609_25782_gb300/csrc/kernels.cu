@@ -739,11 +739,16 @@ __global__ void table_write_kernel(const __grid_constant__ TableWriteArgs a) {
 __global__ void gather_tables_kernel(const __grid_constant__ GatherArgs a) {
     const int r = blockIdx.x;
     if (r >= a.count) return;
-    const int32_t *src = a.arena + static_cast<int64_t>(a.sids[r]) * a.stride;
+    int32_t *src = a.arena + static_cast<int64_t>(a.sids[r]) * a.stride;
     int32_t *dst = a.tables + static_cast<int64_t>(a.row0 + r) * a.max_blocks;
     const int n = a.nblk[r];
-    for (int e = threadIdx.x; e < a.max_blocks; e += blockDim.x) dst[e] = e < n ? src[e] : -1;
-    if (threadIdx.x == 0) a.seq_lens[a.row0 + r] = a.lens[r];
+    const int32_t nb = a.new_blk[r];   // a block the row just gained, not yet in the arena
+    for (int e = threadIdx.x; e < a.max_blocks; e += blockDim.x)
+        dst[e] = e < n ? (e == n - 1 && nb >= 0 ? nb : src[e]) : -1;
+    if (threadIdx.x == 0) {
+        if (nb >= 0) src[n - 1] = nb;
+        a.seq_lens[a.row0 + r] = a.lens[r];
+    }
 }
 
 }  // namespace

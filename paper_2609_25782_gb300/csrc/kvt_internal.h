@@ -134,7 +134,7 @@ struct TableWriteArgs {
 
 constexpr int kGatherMax = 512;
 struct GatherArgs {
-    const int32_t *arena;     // [max_sessions][stride]
+    int32_t *arena;           // [max_sessions][stride]
     int64_t stride;
     int32_t *tables;          // [B][max_blocks]
     int32_t *seq_lens;
@@ -144,6 +144,7 @@ struct GatherArgs {
     int32_t sids[kGatherMax];
     int32_t lens[kGatherMax];
     int32_t nblk[kGatherMax];
+    int32_t new_blk[kGatherMax];   // >= 0: also store it as the row's last entry (nblk-1)
 };
 
 // Host launchers (kernels.cu). Each returns the launch's CUDA status.

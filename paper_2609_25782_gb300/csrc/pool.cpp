@@ -1005,8 +1005,12 @@ int session_block_table(kv_pool *p, int32_t sid, int32_t *host_row, int32_t cap,
 
 // Device inputs of a decode batch from the pool's tables: row b of
 // block_tables (entries past the session's length set to -1) and seq_lens.
+// lens / nblk / new_blk, when given, replace the sessions' current lengths
+// and row sizes (a call that launches before committing its host state).
 static int gather_batch(kv_pool *p, const int32_t *sids, int32_t B, int32_t *block_tables,
-                        int32_t max_blocks, int32_t *seq_lens, cudaStream_t st) {
+                        int32_t max_blocks, int32_t *seq_lens, cudaStream_t st,
+                        const int32_t *lens = nullptr, const int32_t *nblk = nullptr,
+                        const int32_t *new_blk = nullptr) {
     for (int32_t r0 = 0; r0 < B; r0 += kvt::kGatherMax) {
         kvt::GatherArgs a;
         a.arena = p->d_tables;
@@ -1019,8 +1023,9 @@ static int gather_batch(kv_pool *p, const int32_t *sids, int32_t B, int32_t *blo
         for (int32_t i = 0; i < a.count; ++i) {
             const Session &s = p->sessions[sids[r0 + i]];
             a.sids[i] = sids[r0 + i];
-            a.lens[i] = static_cast<int32_t>(s.T);
-            a.nblk[i] = static_cast<int32_t>(s.blocks.size());
+            a.lens[i] = lens ? lens[r0 + i] : static_cast<int32_t>(s.T);
+            a.nblk[i] = nblk ? nblk[r0 + i] : static_cast<int32_t>(s.blocks.size());
+            a.new_blk[i] = new_blk ? new_blk[r0 + i] : -1;
         }
         int rc = p->cuda("gather launch", [&] { return kvt::launch_gather(a, st); });
         if (rc) return rc;
@@ -1127,10 +1132,21 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
     if (!rc && !fresh.empty()) rc = p->wait_fences(fresh.data(), fresh.size(), st);
     if (!rc) rc = p->evict_device(vic, st);
     if (!rc) rc = p->run_jobs(jobs, false, st);
+    // A row that only grew gets its new entry from the gather launch below
+    // (host-logic pools gather nothing and write no device rows).
+    std::vector<int32_t> new_blk(B, -1), lens(B), nblk(B);
     for (int32_t i = 0; !rc && i < B; ++i) {
         const int64_t n = static_cast<int64_t>(rows[i].size()) - first[i];
-        if (n > 0) rc = p->write_table(sids[i], rows[i].data() + first[i], first[i], n, st);
+        if (n == 1 && miss[i].empty())
+            new_blk[i] = rows[i].back();
+        else if (n > 0)
+            rc = p->write_table(sids[i], rows[i].data() + first[i], first[i], n, st);
+        lens[i] = static_cast<int32_t>(p->sessions[sids[i]].T + 1);
+        nblk[i] = static_cast<int32_t>(rows[i].size());
     }
+    if (!rc && !p->host_only)
+        rc = gather_batch(p, sids, B, block_tables, max_blocks, seq_lens, st, lens.data(),
+                          nblk.data(), new_blk.data());
     if (rc) return rc;   // host state untouched
 
     p->evict_commit(vic);
@@ -1154,8 +1170,7 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
     p->stats.bytes_unpacked += fetched * p->token_bytes;
     p->stats.bytes_appended += static_cast<int64_t>(B) * p->token_bytes;
     p->stats.appends += B;
-    if (p->host_only) return KV_OK;
-    return gather_batch(p, sids, B, block_tables, max_blocks, seq_lens, st);
+    return KV_OK;
 }
 
 int kv_pool_shuffle_free(kv_pool *p, uint64_t seed) {
