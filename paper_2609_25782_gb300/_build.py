@@ -1,8 +1,8 @@
 """Compile libkvtier.so in-tree with nvcc for sm_103a.
 
-The translation units (kernels.cu, pool.cpp, noalloc.cu) compile in parallel and are
-linked with the static CUDA runtime, so the library needs only the driver at
-run time.
+The translation units (decode_kernels.cu, copy_kernels.cu, pool.cpp,
+noalloc.cu) compile in parallel and are linked with the static CUDA runtime,
+so the library needs only the driver at run time.
 """
 from __future__ import annotations
 
@@ -14,7 +14,7 @@ import sys
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libkvtier.so")
-SOURCES = ["kernels.cu", "pool.cpp", "noalloc.cu"]
+SOURCES = ["decode_kernels.cu", "copy_kernels.cu", "pool.cpp", "noalloc.cu"]
 HEADERS = ["kvt_internal.h", os.path.join("..", "..", "include", "kvtier.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -1,5 +1,5 @@
 // Internal interface between the pool runtime (pool.cpp) and the kernels
-// (kernels.cu). Not part of the C ABI.
+// (decode_kernels.cu, copy_kernels.cu). Not part of the C ABI.
 #pragma once
 
 #include <cuda.h>
@@ -147,7 +147,7 @@ struct GatherArgs {
     int32_t new_blk[kGatherMax];   // >= 0: also store it as the row's last entry (nblk-1)
 };
 
-// Host launchers (kernels.cu). Each returns the launch's CUDA status.
+// Host launchers (decode_kernels.cu, copy_kernels.cu). Each returns the launch's CUDA status.
 bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why);
 cudaError_t prepare_kernels();  // per-device function attributes
 // overlap_previous: launch the split kernel as a programmatic dependent of the

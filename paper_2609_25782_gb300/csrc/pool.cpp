@@ -4,7 +4,8 @@
 // paper): the hot free list and per-session block tables, the cold-arena
 // placement of per-session images, the session states {ACTIVE, PAUSED}, the
 // write-on-evict watermark (cold_valid), and the CUDA events that order
-// migrations against decode. Device work goes to the kernels in kernels.cu.
+// migrations against decode. Device work goes to the kernels in
+// decode_kernels.cu and copy_kernels.cu.
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
