@@ -707,6 +707,21 @@ def cpu_baseline(res, seed, budget_s=15.0):
                       f"fp64 CPU oracle, {spent:.1f} s"}
 
 
+METRIC = "decode-attn KV GB/s (per step over all layers; resume-unpack GB/s and ms in secondary)"
+
+
+def workload_name(args) -> str:
+    """The decode workload's name, shared by both arms' JSON lines."""
+    nl, nbatch = args.layers, args.batch
+    if (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2):
+        shape = ("Qwen3-Coder-30B-A3B KV shape (48 layers, Hq 32, Hkv 4, D 128, 16-token blocks), "
+                 "32 sessions with contexts U[8K,32K]")
+    else:
+        shape = (f"{nl} layers (Hq 32, Hkv 4, D 128, 16-token blocks), {nbatch} sessions with "
+                 f"contexts U[{args.tmin},{args.tmax}] (reduced profiling case)")
+    return f"decode-attention step: {shape}, random physical blocks"
+
+
 def run_reference(args):
     """The oracle timed as the reference arm on host cores: each step is one
     layer of four sessions of the decode workload (lengths from the same
@@ -730,12 +745,12 @@ def run_reference(args):
     kv = int(np.sum(lens)) * 2 * HKV * D * 2 * args.steps
     val = kv / dt / 1e9
     line = {
-        "impl": "reference", "metric": "decode-attn KV GB/s", "value": round(val, 4), "unit": "GB/s",
+        "impl": "reference", "metric": METRIC, "value": round(val, 4), "unit": "GB/s",
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": "decode-attention step, Qwen3-Coder-30B-A3B KV shape, 32 sessions "
-                               "x [8K,32K] tokens; each reference step: layer 0 of 4 sessions"},
+        "config": {"workload": workload_name(args),
+                   "reference_step": "the CPU oracle on layer 0 of 4 of the sessions (bounded sample)"},
         "cpu_baseline": {"value": round(val, 4), "unit": "GB/s", "cores": oracle.threads(),
                          "kind": "oracle",
                          "sample": f"layer 0 of 4 sessions ({int(np.sum(lens))} tokens) per step"},
@@ -846,20 +861,16 @@ def main():
         secondary["trace_lru"] = run_trace(args, rank, lru_factor=1.5)
     nl, nbatch = args.layers, args.batch
     headline = (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2)
-    shape = ("Qwen3-Coder-30B-A3B KV shape (48 layers, Hq 32, Hkv 4, D 128, 16-token blocks), "
-             "32 sessions with contexts U[8K,32K]" if headline else
-             f"{nl} layers (Hq 32, Hkv 4, D 128, 16-token blocks), {nbatch} sessions with contexts "
-             f"U[{args.tmin},{args.tmax}] (reduced profiling case)")
 
     if rank == 0:
         line = {
-            "metric": "decode-attn KV GB/s (per step over all layers; resume-unpack GB/s and ms in secondary)",
+            "metric": METRIC,
             "value": round(value, 1), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
             "config": {
-                "workload": f"decode-attention step: {shape}, random physical blocks",
+                "workload": workload_name(args),
                 "tokens": int(np.sum(res["lens"])), "kv_gb_per_step": round(res["kv_bytes"] / 1e9, 2),
                 "launches_per_step": res["launches_per_call"] * nl, "compute": "bf16 inputs, fp32 softmax/accumulate",
                 "cuda_graph": res["graph"],
