@@ -888,7 +888,8 @@ def main():
                                    "(timed region / calls)",
                          "alg_bytes_per_launch": int(res["launch_alg_bytes"])},
             "cpu_baseline": cpu,
-            "gpu_launches": res["launches_per_call"] * nl * args.steps,
+            # every rank launches the same per-step kernels; whole-job count, like `value`
+            "gpu_launches": res["launches_per_call"] * nl * args.steps * ws,
             "clocks": res["clocks"],
             "secondary": secondary,
         }
