@@ -134,6 +134,8 @@ __global__ void __launch_bounds__(256) block_jobs_kernel(const __grid_constant__
             if (lane == 0 && ch == 0 && c == 0) atomicOr(a.err, kErrBadBlock);
             continue;
         }
+        if (!kPack && b.sid >= 0 && c == 0 && ch == 0 && lane == 0)   // a fetch: its table entry
+            a.tables[static_cast<int64_t>(b.sid) * a.table_stride + b.j] = b.slot;
         const int t_lo = max(b.t0, ch * kMigChunkTokens);
         const int t_hi = min(b.t1, (ch + 1) * kMigChunkTokens);
         if (t_hi <= t_lo) continue;

@@ -112,13 +112,16 @@ struct AppendArgs {
 // logical block j (all layers, K and V, all kv-heads).
 struct BlockJob {
     uint8_t *img;             // the session's image base
-    int64_t T_cap;
+    int32_t T_cap;            // image rows per (layer, K|V, kv-head) run (contexts <= 2^30)
+    int32_t sid;              // a fetch: the session whose table entry j becomes `slot`; -1: none
     int32_t slot, j, t0, t1;
 };
 constexpr int kBlockJobsMax = 960;   // keeps the parameter block under 32 KB
 struct BlockJobs {
     uint8_t *hot;
     int32_t *err;
+    int32_t *tables;          // the pool's table arena (fetch jobs write their entry)
+    int64_t table_stride;
     Shape s;
     int32_t n;
     int32_t pad;

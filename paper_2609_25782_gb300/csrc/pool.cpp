@@ -307,11 +307,20 @@ struct kv_pool {
         const Session &s = sessions[sid];
         kvt::BlockJob b;
         b.img = static_cast<uint8_t *>(cfg.cold_base) + s.img_off;
-        b.T_cap = s.cap;
+        b.T_cap = static_cast<int32_t>(s.cap);
+        b.sid = -1;
         b.slot = slot;
         b.j = j;
         b.t0 = t0;
         b.t1 = t1;
+        return b;
+    }
+
+    // A fetch of block j into `slot`: the copy also writes the session's
+    // device table entry j.
+    kvt::BlockJob fetch_job(int32_t sid, int32_t j, int32_t slot, int32_t t0, int32_t t1) const {
+        kvt::BlockJob b = job_for(sid, j, slot, t0, t1);
+        b.sid = sid;
         return b;
     }
 
@@ -320,6 +329,8 @@ struct kv_pool {
             kvt::BlockJobs a;
             a.hot = static_cast<uint8_t *>(cfg.hot_base);
             a.err = d_err;
+            a.tables = d_tables;
+            a.table_stride = table_stride;
             a.s = shape;
             a.n = static_cast<int32_t>(std::min<size_t>(kvt::kBlockJobsMax, jobs.size() - i));
             a.pad = 0;
@@ -575,9 +586,8 @@ static int lru_append(kv_pool *p, int32_t sid, const void *k, const void *v, int
     if (!rc && s->ready_recorded) rc = wait_event(p, st, s->ready);
     if (!rc) rc = p->evict_device(vic, st);
     if (!rc && refetch) {
-        rc = p->run_jobs({p->job_for(sid, static_cast<int32_t>(tail), got[0], 0,
-                                     p->tokens_in_block(*s, tail))}, false, st);
-        if (!rc) rc = p->write_table(sid, &got[0], tail, 1, st);
+        rc = p->run_jobs({p->fetch_job(sid, static_cast<int32_t>(tail), got[0], 0,
+                                       p->tokens_in_block(*s, tail))}, false, st);
     }
     if (!rc && fresh_n > 0)
         rc = p->write_table(sid, got.data() + (refetch ? 1 : 0), have, fresh_n, st);
@@ -638,7 +648,7 @@ static int lru_resume(kv_pool *p, int32_t sid, cudaStream_t st) {
     for (int64_t i = 0; i < need; ++i) {
         const int32_t j = missing[i];
         row[j] = got[i];
-        jobs.push_back(p->job_for(sid, j, got[i], 0, p->tokens_in_block(*s, j)));
+        jobs.push_back(p->fetch_job(sid, j, got[i], 0, p->tokens_in_block(*s, j)));
         fetched += p->tokens_in_block(*s, j);
     }
 
@@ -646,7 +656,6 @@ static int lru_resume(kv_pool *p, int32_t sid, cudaStream_t st) {
     int rc = ensure_event(p, &s->ready);
     if (!rc) rc = p->evict_device(vic, st);
     if (!rc) rc = p->run_jobs(jobs, false, st);
-    if (!rc && need > 0) rc = p->write_table(sid, row.data(), 0, static_cast<int64_t>(row.size()), st);
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
     if (rc) return rc;
 
@@ -695,16 +704,13 @@ static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStrea
         rows[u] = s.blocks;
         for (int32_t j : miss[u]) {
             rows[u][j] = got[k];
-            jobs.push_back(p->job_for(uniq[u], j, got[k], 0, p->tokens_in_block(s, j)));
+            jobs.push_back(p->fetch_job(uniq[u], j, got[k], 0, p->tokens_in_block(s, j)));
             fetched += p->tokens_in_block(s, j);
             ++k;
         }
     }
     int rc = p->evict_device(vic, st);
-    if (!rc) rc = p->run_jobs(jobs, false, st);
-    for (size_t u = 0; !rc && u < uniq.size(); ++u)
-        if (!miss[u].empty())
-            rc = p->write_table(uniq[u], rows[u].data(), 0, static_cast<int64_t>(rows[u].size()), st);
+    if (!rc) rc = p->run_jobs(jobs, false, st);   // the fetches also write their table entries
     if (rc) return rc;
 
     p->evict_commit(vic);
@@ -1101,19 +1107,16 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
         return fail(KV_ERR_NO_HOT_BLOCKS, "the batch's blocks and new positions do not fit in the hot pool");
     const std::vector<int32_t> got = p->peek_alloc(need, vic);
     std::vector<std::vector<int32_t>> rows(B);
-    std::vector<int64_t> first(B);   // first changed table entry per member
     std::vector<kvt::BlockJob> jobs;
     std::vector<int32_t> fresh;      // popped slots that are not eviction victims
     int64_t k = 0, fetched = 0;
     for (int32_t i = 0; i < B; ++i) {
         const Session &s = p->sessions[sids[i]];
         rows[i] = s.blocks;
-        first[i] = static_cast<int64_t>(s.blocks.size());
         for (int32_t j : miss[i]) {
             rows[i][j] = got[k];
-            jobs.push_back(p->job_for(sids[i], j, got[k], 0, p->tokens_in_block(s, j)));
+            jobs.push_back(p->fetch_job(sids[i], j, got[k], 0, p->tokens_in_block(s, j)));
             fetched += p->tokens_in_block(s, j);
-            first[i] = std::min<int64_t>(first[i], j);
             ++k;
         }
         if (grow[i]) rows[i].push_back(got[k++]);
@@ -1133,15 +1136,11 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
     if (!rc && !fresh.empty()) rc = p->wait_fences(fresh.data(), fresh.size(), st);
     if (!rc) rc = p->evict_device(vic, st);
     if (!rc) rc = p->run_jobs(jobs, false, st);
-    // A row that only grew gets its new entry from the gather launch below
-    // (host-logic pools gather nothing and write no device rows).
+    // Fetched entries were written by their jobs; a new tail block's entry is
+    // written by the gather launch below (host-logic pools launch nothing).
     std::vector<int32_t> new_blk(B, -1), lens(B), nblk(B);
-    for (int32_t i = 0; !rc && i < B; ++i) {
-        const int64_t n = static_cast<int64_t>(rows[i].size()) - first[i];
-        if (n == 1 && miss[i].empty())
-            new_blk[i] = rows[i].back();
-        else if (n > 0)
-            rc = p->write_table(sids[i], rows[i].data() + first[i], first[i], n, st);
+    for (int32_t i = 0; i < B; ++i) {
+        if (grow[i]) new_blk[i] = rows[i].back();
         lens[i] = static_cast<int32_t>(p->sessions[sids[i]].T + 1);
         nblk[i] = static_cast<int32_t>(rows[i].size());
     }
