@@ -943,7 +943,9 @@ int session_resume(kv_pool *p, int32_t sid, kv_stream_t stream_) {
     if (!rc && s->pack_fence >= 0 && p->fences[s->pack_fence].gen == s->pack_gen)
         rc = p->cuda("cudaStreamWaitEvent",
                      [&] { return cudaStreamWaitEvent(st, p->fences[s->pack_fence].ev, 0); });
-    if (!rc && need <= kvt::kResumeInlineMax) {
+    if (!rc && need == 0) {
+        // an empty session: no blocks, nothing to copy
+    } else if (!rc && need <= kvt::kResumeInlineMax) {
         // one launch: the block ids ride in the parameters, the kernel writes the row
         kvt::ResumeArgs r;
         r.m = p->mig_args(sid, *s);

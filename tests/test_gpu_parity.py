@@ -369,6 +369,42 @@ def test_incremental_pack_resume_bit_exact(pkg, bt, T1, T2):
     pool.close()
 
 
+def test_empty_session_pause_resume(pkg):
+    """A session with no tokens pauses and resumes (nothing to move; the only
+    way to have an empty paused session), then takes tokens and decodes like
+    any other."""
+    dev = torch.device("cuda:0")
+    L = 2
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=16, cold_bytes=1 << 24, max_sessions=3,
+                    max_batch=4, max_context=256)
+    a = pool.session_create(256)
+    b = pool.session_create(256)
+    for s in (a, b):
+        pool.session_pause(s)
+        pool.session_resume(s)
+    for s in (a, b):
+        assert pool.session_block_table(s) == [] and int(pool.session_info(s).tokens) == 0
+        k, v = synth.kv_logical_torch(5, s, range(L), 4, 128, 0, 20, dev)
+        pool.session_append(s, k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous())
+    tables = torch.empty(2, 16, dtype=torch.int32, device=dev)
+    lens = torch.empty(2, dtype=torch.int32, device=dev)
+    pool.batch_tables([a, b], tables, 16, lens)
+    q = synth.queries_torch(5, [a, b], range(L), 32, 128, dev)
+    out = torch.empty(L, 2, 32, 128, dtype=torch.float32, device=dev)
+    pool.decode_attention(-1, q, tables, lens, 2, 16, 1 / math.sqrt(128), out)
+    torch.cuda.synchronize()
+    rows = np.full((2, 16), -1, dtype=np.int32)
+    for r, s in enumerate((a, b)):
+        row = pool.session_block_table(s)
+        rows[r, :len(row)] = row
+    hot = synth.hot_pool_np(5, [a, b], [20, 20], rows, 16, L, 4, 128, 16)
+    ref = oracle.paged_decode(hot, q.cpu().view(torch.int16).numpy().view(np.uint16), rows,
+                              [20, 20], 1 / math.sqrt(128), 32)
+    assert scaled_err(out.cpu().double().numpy(), ref) <= TOL
+    assert pool.check_device() == 0
+    pool.close()
+
+
 def test_config1_scenario(pkg):
     """Tiny single-layer case: 4 sessions (512..2048 tokens, one partial tail)
     decode; a 5th 1024-token session is packed, its blocks freed, the free
