@@ -413,6 +413,8 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
     p->sessions.resize(c.max_sessions);
     if (c.cold_bytes > 0) p->cold_free[0] = c.cold_bytes;
 
+    // decode workspace capacity (also checked against calls on host-logic pools)
+    p->part_rows = static_cast<int64_t>(c.max_batch) * c.num_q_heads * p->max_splits;
     if (!host_only) {
         DeviceGuard dg(c.device, true);
         auto bail = [&](int rc) {
@@ -423,8 +425,7 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
             return bail(fail(KV_ERR_CUDA, "cudaSetDevice failed"));
         cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, c.device);
         const int64_t tbl = static_cast<int64_t>(c.max_sessions) * p->table_stride * 4;
-        const int64_t prow = static_cast<int64_t>(c.max_batch) * c.num_q_heads * p->max_splits;
-        p->part_rows = prow;
+        const int64_t prow = p->part_rows;
         int rc = p->cuda("cudaMalloc(tables)", [&] { return cudaMalloc(&p->d_tables, tbl); });
         if (!rc) rc = p->cuda("cudaMalloc(partials)", [&] {
             return cudaMalloc(&p->d_part_o, prow * kvt::kHeadDim * sizeof(float));
@@ -803,7 +804,6 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
     if (!q || !block_tables || !seq_lens || !out) return fail(KV_ERR_INVALID_ARG, "null pointer");
     if (!decode_pointers_aligned(q, block_tables, seq_lens, out))
         return fail(KV_ERR_INVALID_ARG, "q, block_tables, seq_lens need 4-byte and out 16-byte alignment");
-    if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
     if (layer < -1 || layer >= p->cfg.num_layers) return fail(KV_ERR_INVALID_ARG, "bad layer");
     const int nl = layer < 0 ? p->cfg.num_layers : 1;
     if (B < 1 || static_cast<int64_t>(nl) * B > 65535)
@@ -817,6 +817,8 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
                     "decode workspace too small: layers x B x Hq x splits(max_blocks) exceeds "
                     "max_batch x Hq x splits(max_context)");
     if (!(scale == scale) || std::isinf(scale)) return fail(KV_ERR_INVALID_ARG, "scale not finite");
+    // arguments first, then the pool's state
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "decode_attention on a host-logic-only pool");
     DeviceGuard dg(p->cfg.device, true);
     kvt::DecodeArgs a;
     a.q = static_cast<const uint16_t *>(q);

@@ -222,3 +222,32 @@ def test_bad_configs_rejected(kv):
         assert e.value.code == kv.KV_ERR_INVALID_ARG
     with pytest.raises(kv.KVError):   # real pools need arenas
         kv.kv_pool_create(kv.make_config(num_layers=2, num_hot_blocks=10))
+
+
+def test_decode_arguments_checked_before_any_launch(kv):
+    """Every argument of a decode call is validated before the pool's state
+    (a host-logic pool then refuses to compute): layer, batch size, table
+    width, the workspace the call needs, the scale."""
+    cfg = kv.make_config(num_layers=4, num_hot_blocks=64, max_batch=2, max_context=1024,
+                         flags=kv.KV_POOL_HOST_LOGIC_ONLY)
+    pool = kv.kv_pool_create(cfg)
+    q, tab, lens, out = 256, 512, 768, 1024            # aligned stand-ins, never dereferenced
+    cases = [
+        dict(layer=4), dict(layer=-2), dict(B=0), dict(B=65536), dict(layer=-1, B=16384),
+        dict(max_blocks=0), dict(max_blocks=(1 << 26) + 1),
+        dict(max_blocks=1024),                  # 16K-token tables: 16 splits x 32 heads > 2 x 32 x 1
+        dict(layer=-1, B=2),                    # 4 layers x 2 rows x 32 heads > 64 rows
+        dict(scale=float("nan")), dict(scale=float("inf")),
+    ]
+    for c in cases:
+        a = dict(layer=0, B=1, max_blocks=64, scale=1.0) | c
+        with pytest.raises(kv.KVError) as e:
+            kv.decode_attention(pool, a["layer"], q, tab, lens, a["B"], a["max_blocks"], a["scale"],
+                                out, None)
+        assert e.value.code == kv.KV_ERR_INVALID_ARG, c
+    for ok in (dict(layer=0, B=2, max_blocks=64), dict(layer=3, B=1, max_blocks=64)):
+        with pytest.raises(kv.KVError) as e:    # valid arguments: the pool cannot compute
+            kv.decode_attention(pool, ok["layer"], q, tab, lens, ok["B"], ok["max_blocks"], 1.0,
+                                out, None)
+        assert e.value.code == kv.KV_ERR_BAD_STATE, ok
+    kv.kv_pool_destroy(pool)
