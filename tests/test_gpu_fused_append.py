@@ -188,3 +188,38 @@ def test_fused_argument_errors(pkg):
     assert pool.check_device() == 0
     assert torch.all(out == 0)     # one token of zeros: softmax weight 1 on a zero V row
     pool.close()
+
+
+def test_fused_step_bf16_output(pkg):
+    """The fused step writing bf16 output gives the fp32 fused result rounded
+    to nearest even, and the same pool contents."""
+    dev = torch.device("cuda:0")
+    lens = [15, 16, 300, 3000]
+    outs = []
+    for dtype in (torch.float32, torch.bfloat16):
+        L, B, bt = 2, len(lens), 16
+        cap = max(lens) + 2
+        pool = pkg.Pool(num_layers=L, num_hot_blocks=sum(-(-(t + 1) // bt) for t in lens) + 8,
+                        cold_bytes=B * (cap * L * 2 * HKV * D * 2 + 256), max_sessions=B,
+                        max_batch=L * B, max_context=cap, alloc_seed=5)
+        sids = [pool.session_create(cap) for _ in lens]
+        for sid, t in zip(sids, lens):
+            k, v = synth.kv_logical_torch(SEED, sid, range(L), HKV, D, 0, t, dev)
+            pool.session_append(sid, k.permute(0, 2, 1, 3).contiguous(),
+                                v.permute(0, 2, 1, 3).contiguous())
+        q = synth.queries_torch(SEED, sids, range(L), HQ, D, dev)
+        mb = -(-cap // bt)
+        tables = torch.empty(B, mb, dtype=torch.int32, device=dev)
+        slens = torch.empty(B, dtype=torch.int32, device=dev)
+        kn, vn = token_rows(sids, lens, L, dev)
+        pool.batch_reserve(sids, tables, mb, slens)
+        out = torch.empty(L, B, HQ, D, dtype=dtype, device=dev)
+        for l in range(L):
+            pool.decode_append_attention(l, q[l], kn[l], vn[l], tables, slens, B, mb,
+                                         1 / math.sqrt(D), out[l], overlap_previous=l > 0)
+        torch.cuda.synchronize()
+        assert pool.check_device() == 0
+        outs.append(out.cpu())
+        check_pool_holds_sessions(pool, sids, [t + 1 for t in lens], L, bt)
+        pool.close()
+    assert torch.equal(outs[0].to(torch.bfloat16).view(torch.int16), outs[1].view(torch.int16))
