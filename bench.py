@@ -567,7 +567,7 @@ def run_sweep(args):
     KV <= 120 GB, per-layer launches and the all-layers launch."""
     import torch
     import synth
-    from paper_2609_25782_gb300 import Pool
+    from paper_2609_25782_gb300 import Pool, kvtier
     dev = torch.device("cuda", torch.cuda.current_device())
     peak, _ = hbm_peak()
     # resume-unpack sweep (first, before the long decode sweep loads the GPU)
@@ -611,9 +611,8 @@ def run_sweep(args):
         max_tok = max(B * T for B, T in pts)
         nb = max_tok // bt + 64
         Bmax = max(B for B, _ in pts)
-        # workspace rows: the largest of layers x B x Hq x splits(T) over the points
-        def splits(t):    # the library's split bound for t tokens
-            return max(-(-t // 2048), min(16, -(-t // 1024)))
+        # workspace rows: the largest of layers x B x Hq x S(T) over the points
+        splits = kvtier.kv_decode_splits
         need = max(L * B * HQ * splits(T) for B, T in pts)
         ctx = max(SWEEP_T)
         pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,

@@ -151,6 +151,13 @@ int64_t kv_block_bytes(const kv_pool_config *cfg);
  * model, Section 4). */
 int64_t kv_token_bytes(const kv_pool_config *cfg);
 
+/* S(t): the most KV splits a decode call makes for one (session, head) of up
+ * to t tokens, the factor by which the decode workspace scales (see
+ * decode_attention). Each session of T tokens is cut into ceil(T/16) 16-token
+ * tiles and split every clamp(ceil(tiles/16), 64, 128) tiles, a function of T
+ * alone. Returns 0 for t < 1. */
+int32_t kv_decode_splits(int64_t t);
+
 /* Create an ACTIVE, empty session able to hold max_tokens (1 ..
  * max_context) tokens; reserves its cold image (max_tokens * token bytes)
  * in the cold arena (first fit). Errors: KV_ERR_NO_COLD_SPACE, too many
@@ -195,9 +202,9 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  * The result depends only on the values and seq_lens: not on physical
  * placement, batch composition or timing (bit-identical across a
  * pause/resume round trip). The pool's decode workspace holds
- * max_batch x Hq x S(max_context) partial rows, S(t) being the split bound
- * for t tokens (ceil(t / 1024) up to 16 splits, ceil(t / 2048) beyond 32K
- * tokens); a call needs
+ * max_batch x Hq x S(max_context) partial rows, S(t) = kv_decode_splits(t)
+ * (ceil(t / 1024) up to 16 splits, ceil(t / 2048) beyond 32K tokens); a
+ * call needs
  * layers x B x Hq x S(max_blocks x bt) rows, else KV_ERR_INVALID_ARG. Calls on
  * one pool share the workspace: issue them in order on one stream. */
 int decode_attention(kv_pool *pool, int32_t layer, const void *q,

@@ -368,6 +368,10 @@ int64_t kv_block_bytes(const kv_pool_config *c) {
     return c ? kv_token_bytes(c) * c->block_tokens : 0;
 }
 
+int32_t kv_decode_splits(int64_t t) {
+    return t < 1 ? 0 : kvt::max_splits_for(t);
+}
+
 int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
     if (!cfg || !out) return fail(KV_ERR_INVALID_ARG, "kv_pool_create: null argument");
     const kv_pool_config &c = *cfg;

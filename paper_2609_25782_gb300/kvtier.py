@@ -38,7 +38,7 @@ EXPORTS = [
     "kv_pool_free_list", "kv_pool_get_stats", "kv_pool_check_device",
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
     "decode_attention_ex", "kv_pool_set_migration_limit", "kv_pool_batch_reserve",
-    "decode_append_attention", "kv_pool_inject_decode_timeout",
+    "decode_append_attention", "kv_pool_inject_decode_timeout", "kv_decode_splits",
 ]
 
 KV_DEVICE_BAD_BLOCK, KV_DEVICE_BAD_LENGTH, KV_DEVICE_TIMEOUT = 1, 2, 4
@@ -91,6 +91,7 @@ def _load():
         "kv_pool_destroy": [p],
         "kv_block_bytes": [C.POINTER(kv_pool_config)],
         "kv_token_bytes": [C.POINTER(kv_pool_config)],
+        "kv_decode_splits": [i64],
         "session_create": [p, i64, C.POINTER(i32)],
         "session_create_paused": [p, i64, i64, C.POINTER(i32)],
         "session_destroy": [p, i32],
@@ -164,6 +165,11 @@ def kv_token_bytes(cfg: kv_pool_config) -> int:
 
 def kv_block_bytes(cfg: kv_pool_config) -> int:
     return int(lib.kv_block_bytes(C.byref(cfg)))
+
+
+def kv_decode_splits(t: int) -> int:
+    """Most KV splits a decode call makes per (session, head) for up to t tokens."""
+    return int(lib.kv_decode_splits(t))
 
 
 def kv_pool_create(cfg: kv_pool_config) -> int:

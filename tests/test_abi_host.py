@@ -43,6 +43,21 @@ def test_sizes_match_paper_shape(kv):
     assert kv.kv_block_bytes(cfg) == 1536 * 1024
 
 
+def test_decode_split_bound(kv):
+    """S(t) is the tight bound of the per-session split count over T <= t, for
+    splits of clamp(ceil(tiles/16), 64, 128) 16-token tiles."""
+    import numpy as np
+    T = np.arange(1, 140_001)
+    tiles = -(-T // 16)
+    st = np.clip(-(-tiles // 16), 64, 128)
+    running = np.maximum.accumulate(-(-tiles // st))
+    for t in (1, 1024, 1025, 4096, 16384, 16385, 32768, 32769, 65536, 131072, 140000):
+        assert kv.kv_decode_splits(t) == running[t - 1], t
+    assert [kv.kv_decode_splits(t) for t in (1024, 1025, 16384, 32768, 32769, 131072)] == \
+        [1, 2, 16, 16, 17, 64]
+    assert kv.kv_decode_splits(0) == 0 and kv.kv_decode_splits(-5) == 0
+
+
 def host_pool(kv, nb=40, seed=7, L=2, bt=16, cold_tokens=10000, max_sessions=8, max_context=4096):
     cfg = kv.make_config(num_layers=L, num_hot_blocks=nb, block_tokens=bt, alloc_seed=seed,
                          max_sessions=max_sessions, max_context=max_context,
