@@ -48,13 +48,26 @@ def hbm_peak():
         return FALLBACK_HBM, "fallback"
 
 
+TRAFFIC_RECORD = "decode_split_kernel_traffic_48L_B32_8K-32K.txt"
+
+
 def recorded_traffic():
     """DRAM bytes per launch of the decode split kernel from the committed ncu
     capture, or None when the kernel source changed since it was taken."""
     try:
-        with open(os.path.join(ROOT, "profiles", "decode_split_kernel.traffic.json")) as f:
-            rec = json.load(f)
-        for path, sha in rec["sources_sha256"].items():
+        rec, shas = {}, {}
+        with open(os.path.join(ROOT, "profiles", TRAFFIC_RECORD)) as f:
+            for line in f:
+                if line.startswith("#") or ": " not in line:
+                    continue
+                key, val = line.rstrip("\n").split(": ", 1)
+                if key.startswith("sha256 "):
+                    shas[key[len("sha256 "):]] = val
+                else:
+                    rec[key] = val
+        if not shas:
+            return None
+        for path, sha in shas.items():
             with open(os.path.join(ROOT, path), "rb") as f:
                 if hashlib.sha256(f.read()).hexdigest() != sha:
                     return None

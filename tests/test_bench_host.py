@@ -85,3 +85,23 @@ def test_reference_arm_prints_contract_line():
 def test_reference_arm_other_ranks_are_silent():
     r = _run(["--impl", "reference", "--steps", "1"], {"RANK": "1", "WORLD_SIZE": "2"})
     assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_traffic_record_goes_null_when_a_source_changes(tmp_path, monkeypatch):
+    """roofline.traffic comes from the committed ncu record only while every
+    kernel source it names still hashes to the captured value."""
+    sys.path.insert(0, ROOT)
+    import hashlib
+    import bench
+    src = tmp_path / "k.cu"
+    src.write_text("kernel v1\n")
+    (tmp_path / "profiles").mkdir()
+    rec = tmp_path / "profiles" / bench.TRAFFIC_RECORD
+    sha = hashlib.sha256(b"kernel v1\n").hexdigest()
+    rec.write_text(f"# capture\nkernel: k\ndram_bytes_per_launch: 1234\nsha256 k.cu: {sha}\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.recorded_traffic() == 1234
+    src.write_text("kernel v2\n")
+    assert bench.recorded_traffic() is None
+    rec.write_text("kernel: k\ndram_bytes_per_launch: 1234\n")   # no hashes: not trusted
+    assert bench.recorded_traffic() is None
