@@ -203,18 +203,27 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
     const int chunk_rows = sh.Hkv * sh.bt;   // rows between K and V runs
 
+    // Block ids of this warp's tiles, fetched together up front: lane t
+    // holds the block of the warp's tile t, so no table load waits in front
+    // of a tile copy (one CTA per SM has no other warps to hide it behind).
+    static_assert((KVT_SPLIT_MAX_TILES + kDecodeWarps - 1) / kDecodeWarps <= 32,
+                  "a warp's tiles of one split must fit one block id per lane");
+    int lane_blk = 0;
+    if (lane < my_tiles)
+        lane_blk = trow[(tile0 + warp + lane * kDecodeWarps) * kTileTokens / sh.bt];
+
     if (lane == 0) {
         for (int i = 0; i < kStages; ++i) mbar_init(bar0 + 8 * i, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncwarp();
 
-    // Producer step (lane 0): tile k of this warp into slot k % kStages.
-    auto issue = [&](int k) {
+    // Producer step (lane 0): tile k of this warp, in block blk, into slot
+    // k % kStages.
+    auto issue = [&](int k, int blk) {
         const int ti = tile0 + warp + k * kDecodeWarps;
         const int tok = ti * kTileTokens;
         const int j = tok / sh.bt;
-        int blk = trow[j];
         if (blk < 0 || blk >= sh.num_blocks) {
             atomicOr(a.err, kErrBadBlock);
             blk = 0;
@@ -232,8 +241,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         tma_load_2d(slot + 2 * kHalfBytes, &map, 0, rowv, bar);
         tma_load_2d(slot + 3 * kHalfBytes, &map, 64, rowv, bar);
     };
-    if (lane == 0)
-        for (int k = 0; k < kStages && k < my_tiles; ++k) issue(k);
+    // The block of tile k, for every lane (k < 32 wherever it is used).
+    auto blk_of = [&](int k) { return __shfl_sync(0xffffffffu, lane_blk, k & 31); };
+#pragma unroll
+    for (int k = 0; k < kStages; ++k) {
+        const int blk = blk_of(k);
+        if (lane == 0 && k < my_tiles) issue(k, blk);
+    }
 
     // Everything above reads only the hot pool, the block table and seq_lens.
     // When this grid is launched as a programmatic dependent (the caller's
@@ -272,73 +286,63 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     const int vrow = (lane & 7) + (lane >> 4) * 8;
     const int vhi = (lane >> 3) & 1;
 
-    for (int k = 0; k < my_tiles; ++k) {
-        const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
-        if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) {
-            fail_k = k;
-            break;
+    // Fused append: token T-1 arrives with this call. Its K and V rows
+    // replace whatever the copy brought for that slot of tile k and are
+    // stored to the reserved pool slot. Lanes 0-15 move K, 16-31 V, 16 B each.
+    auto splice_new = [&](int k, int tok_base) {
+        const int r = T - 1 - tok_base;
+        const int u = lane & 15;
+        const int isv = lane >> 4;
+        const uint4 val = *reinterpret_cast<const uint4 *>(
+            (isv ? a.v_new : a.k_new) +
+            ((static_cast<int64_t>(li) * a.B + b) * sh.Hkv + g) * kHeadDim + u * 8);
+        *reinterpret_cast<uint4 *>(ring + (k % kStages) * kTileBytes + isv * 2 * kHalfBytes +
+                                   (u >> 3) * kHalfBytes + swz(r, u & 7)) = val;
+        const int j = (T - 1) / sh.bt;
+        const int blk = trow[j];
+        if (blk >= 0 && blk < sh.num_blocks) {   // a bad id was flagged by the copy
+            const int64_t row =
+                ((static_cast<int64_t>(blk) * sh.L + l) * 2 * sh.Hkv + g) * sh.bt +
+                (T - 1 - j * sh.bt) + isv * chunk_rows;
+            *reinterpret_cast<uint4 *>(a.hot + row * kHeadDim + u * 8) = val;
         }
-        const int ti = tile0 + warp + k * kDecodeWarps;
-        const int tok_base = ti * kTileTokens;
-
-        if (a.k_new != nullptr && tok_base + kTileTokens >= T) {
-            // Fused append: token T-1 arrives with this call. Its K and V rows
-            // replace whatever the copy brought for that slot and are stored
-            // to the reserved pool slot. Lanes 0-15 move K, 16-31 V, 16 B each.
-            const int r = T - 1 - tok_base;
-            const int u = lane & 15;
-            const int isv = lane >> 4;
-            const uint4 val = *reinterpret_cast<const uint4 *>(
-                (isv ? a.v_new : a.k_new) +
-                ((static_cast<int64_t>(li) * a.B + b) * sh.Hkv + g) * kHeadDim + u * 8);
-            *reinterpret_cast<uint4 *>(ring + (k % kStages) * kTileBytes + isv * 2 * kHalfBytes +
-                                       (u >> 3) * kHalfBytes + swz(r, u & 7)) = val;
-            const int j = (T - 1) / sh.bt;
-            const int blk = trow[j];
-            if (blk >= 0 && blk < sh.num_blocks) {   // a bad id was flagged by the copy
-                const int64_t row =
-                    ((static_cast<int64_t>(blk) * sh.L + l) * 2 * sh.Hkv + g) * sh.bt +
-                    (T - 1 - j * sh.bt) + isv * chunk_rows;
-                *reinterpret_cast<uint4 *>(a.hot + row * kHeadDim + u * 8) = val;
-            }
-            // The slot is refilled by the async proxy later.
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-        }
-
-        // S^T = K . Q^T, two accumulators to shorten the mma chain.
-        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int ks = 0; ks < 8; ks += 2) {
-            uint32_t r0, r1, r2, r3;
-            int u = 2 * ks + khi;
-            ldsm_x4(slot + (u >> 3) * kHalfBytes + swz(krow, u & 7), r0, r1, r2, r3);
-            mma_bf16(sa, r0, r1, r2, r3, qb[ks][0], qb[ks][1]);
-            u = 2 * (ks + 1) + khi;
-            ldsm_x4(slot + (u >> 3) * kHalfBytes + swz(krow, u & 7), r0, r1, r2, r3);
-            mma_bf16(sb, r0, r1, r2, r3, qb[ks + 1][0], qb[ks + 1][1]);
-        }
+        // The slot is refilled by the async proxy later.
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+    };
+    // One k-step (16 dims) of S^T = K . Q^T into acc.
+    auto qk_step = [&](uint32_t slot, int ks, float (&acc)[4]) {
+        uint32_t r0, r1, r2, r3;
+        const int u = 2 * ks + khi;
+        ldsm_x4(slot + (u >> 3) * kHalfBytes + swz(krow, u & 7), r0, r1, r2, r3);
+        mma_bf16(acc, r0, r1, r2, r3, qb[ks][0], qb[ks][1]);
+    };
+    // Logits in log2 units; tokens at or past T are -inf.
+    auto logits = [&](const float (&sa)[4], const float (&sb)[4], int tok_base, float (&x)[4]) {
         const bool v0 = tok_base + (lane >> 2) < T;
         const bool v1 = tok_base + (lane >> 2) + 8 < T;
-        const float x0 = v0 ? (sa[0] + sb[0]) * sl : -INFINITY;
-        const float x1 = v0 ? (sa[1] + sb[1]) * sl : -INFINITY;
-        const float x2 = v1 ? (sa[2] + sb[2]) * sl : -INFINITY;
-        const float x3 = v1 ? (sa[3] + sb[3]) * sl : -INFINITY;
-        float mx0 = fmaxf(x0, x2), mx1 = fmaxf(x1, x3);
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
-        }
+        x[0] = v0 ? (sa[0] + sb[0]) * sl : -INFINITY;
+        x[1] = v0 ? (sa[1] + sb[1]) * sl : -INFINITY;
+        x[2] = v1 ? (sa[2] + sb[2]) * sl : -INFINITY;
+        x[3] = v1 ? (sa[3] + sb[3]) * sl : -INFINITY;
+    };
+    // Online-softmax step of one tile given its column maxima: advances m and
+    // l, returns P (rounded to bf16, as the PV product sees it) and the
+    // factors that rescale the accumulator.
+    auto softmax_step = [&](const float (&x)[4], float mx0, float mx1, uint32_t &p01,
+                            uint32_t &p23, float &al0, float &al1) {
         const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+        al0 = ex2(m0 - mn0);
+        al1 = ex2(m1 - mn1);
         m0 = mn0;
         m1 = mn1;
-        float q0, q1, q2, q3;   // P rounded to bf16, as the PV product sees it
-        const uint32_t p01 = pack_bf16(ex2(x0 - mn0), ex2(x1 - mn1), q0, q1);
-        const uint32_t p23 = pack_bf16(ex2(x2 - mn0), ex2(x3 - mn1), q2, q3);
+        float q0, q1, q2, q3;
+        p01 = pack_bf16(ex2(x[0] - mn0), ex2(x[1] - mn1), q0, q1);
+        p23 = pack_bf16(ex2(x[2] - mn0), ex2(x[3] - mn1), q2, q3);
         l0 = l0 * al0 + q0 + q2;
         l1 = l1 * al1 + q1 + q3;
+    };
+    auto rescale = [&](float al0, float al1) {
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             o[i][0] *= al0;
@@ -346,13 +350,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             o[i][2] *= al0;
             o[i][3] *= al1;
         }
-        const uint32_t pb0 = movmatrix_t(p01);   // P^T tokens 0-7  -> B fragment
-        const uint32_t pb1 = movmatrix_t(p23);   // P^T tokens 8-15
-
-        const uint32_t vslot = slot + 2 * kHalfBytes;
+    };
+    // Last, partial tile: slots past T may hold anything (NaN); P is 0 there
+    // but 0 * NaN is not, so clear those V rows of tile k.
+    auto clear_tail_v = [&](int k, int tok_base) {
         if (tok_base + kTileTokens > T) {
-            // Last, partial tile: slots past T may hold anything (NaN);
-            // P is 0 there but 0 * NaN is not, so clear those V rows.
             const int first_bad = T - tok_base;
             const int units = (kTileTokens - first_bad) * 16;
             uint8_t *vp = ring + (k % kStages) * kTileBytes + 2 * kHalfBytes;
@@ -365,6 +367,40 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             __syncwarp();
         }
+    };
+    auto tile_base = [&](int k) { return (tile0 + warp + k * kDecodeWarps) * kTileTokens; };
+    auto slot_of = [&](int k) { return ring_s + (k % kStages) * kTileBytes; };
+
+    // One tile: scores, softmax, O^T += V^T . P^T. False: its wait timed out.
+    auto one_tile = [&](int k) -> bool {
+        const uint32_t slot = slot_of(k);
+        if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) return false;
+        const int tok_base = tile_base(k);
+        if (a.k_new != nullptr && tok_base + kTileTokens >= T) splice_new(k, tok_base);
+
+        // S^T = K . Q^T, two accumulators to shorten the mma chain.
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 8; ks += 2) {
+            qk_step(slot, ks, sa);
+            qk_step(slot, ks + 1, sb);
+        }
+        float x[4];
+        logits(sa, sb, tok_base, x);
+        float mx0 = fmaxf(x[0], x[2]), mx1 = fmaxf(x[1], x[3]);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+        }
+        uint32_t p01, p23;
+        float al0, al1;
+        softmax_step(x, mx0, mx1, p01, p23, al0, al1);
+        rescale(al0, al1);
+        const uint32_t pb0 = movmatrix_t(p01);   // P^T tokens 0-7  -> B fragment
+        const uint32_t pb1 = movmatrix_t(p23);   // P^T tokens 8-15
+        clear_tail_v(k, tok_base);
+        const uint32_t vslot = slot + 2 * kHalfBytes;
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
             uint32_t r0, r1, r2, r3;
@@ -373,7 +409,92 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             mma_bf16(o[i], r0, r1, r2, r3, pb0, pb1);
         }
         __syncwarp();
-        if (lane == 0 && k + kStages < my_tiles) issue(k + kStages);
+        const int nblk = blk_of(k + kStages);
+        if (lane == 0 && k + kStages < my_tiles) issue(k + kStages, nblk);
+        return true;
+    };
+
+    // Tiles k and k+1 together (one CTA per SM, where each warp's own
+    // dependent mma/shuffle latency is the limit): the two tiles' score
+    // products and column maxima run as independent chains, and tile k+1's V
+    // fragments are loaded before tile k's product lands. The state updates
+    // (m, l, then O) are applied tile k first, exactly as in one_tile, so the
+    // result is bit-identical.
+    auto two_tiles = [&](int k) -> bool {
+        const uint32_t sla = slot_of(k), slb = slot_of(k + 1);
+        if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) return false;
+        if (!mbar_wait(bar0 + 8 * ((k + 1) % kStages), ((k + 1) / kStages) & 1)) return false;
+        const int tba = tile_base(k), tbb = tile_base(k + 1);
+        if (a.k_new != nullptr && tba + kTileTokens >= T) splice_new(k, tba);
+        if (a.k_new != nullptr && tbb + kTileTokens >= T) splice_new(k + 1, tbb);
+        clear_tail_v(k, tba);
+        clear_tail_v(k + 1, tbb);
+
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+        float ta[4] = {0.f, 0.f, 0.f, 0.f}, tb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 8; ks += 2) {
+            qk_step(sla, ks, sa);
+            qk_step(slb, ks, ta);
+            qk_step(sla, ks + 1, sb);
+            qk_step(slb, ks + 1, tb);
+        }
+        float xa[4], xb[4];
+        logits(sa, sb, tba, xa);
+        logits(ta, tb, tbb, xb);
+        float ma0 = fmaxf(xa[0], xa[2]), ma1 = fmaxf(xa[1], xa[3]);
+        float mb0 = fmaxf(xb[0], xb[2]), mb1 = fmaxf(xb[1], xb[3]);
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            ma0 = fmaxf(ma0, __shfl_xor_sync(0xffffffffu, ma0, off));
+            ma1 = fmaxf(ma1, __shfl_xor_sync(0xffffffffu, ma1, off));
+            mb0 = fmaxf(mb0, __shfl_xor_sync(0xffffffffu, mb0, off));
+            mb1 = fmaxf(mb1, __shfl_xor_sync(0xffffffffu, mb1, off));
+        }
+        uint32_t pa01, pa23, pb01, pb23;
+        float ala0, ala1, alb0, alb1;
+        softmax_step(xa, ma0, ma1, pa01, pa23, ala0, ala1);
+        softmax_step(xb, mb0, mb1, pb01, pb23, alb0, alb1);
+        rescale(ala0, ala1);
+        const uint32_t pa0 = movmatrix_t(pa01), pa1 = movmatrix_t(pa23);
+        const uint32_t pb0 = movmatrix_t(pb01), pb1 = movmatrix_t(pb23);
+        uint32_t vb[8][4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            uint32_t r0, r1, r2, r3;
+            const int u = 2 * i + vhi;
+            ldsm_x4_t(sla + 2 * kHalfBytes + (u >> 3) * kHalfBytes + swz(vrow, u & 7), r0, r1, r2,
+                      r3);
+            mma_bf16(o[i], r0, r1, r2, r3, pa0, pa1);
+            ldsm_x4_t(slb + 2 * kHalfBytes + (u >> 3) * kHalfBytes + swz(vrow, u & 7), vb[i][0],
+                      vb[i][1], vb[i][2], vb[i][3]);
+        }
+        rescale(alb0, alb1);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mma_bf16(o[i], vb[i][0], vb[i][1], vb[i][2], vb[i][3], pb0, pb1);
+        __syncwarp();
+        const int nblk0 = blk_of(k + kStages), nblk1 = blk_of(k + 1 + kStages);
+        if (lane == 0) {
+            if (k + kStages < my_tiles) issue(k + kStages, nblk0);
+            if (k + 1 + kStages < my_tiles) issue(k + 1 + kStages, nblk1);
+        }
+        return true;
+    };
+
+    for (int k = 0; k < my_tiles;) {
+        if (kStages == kStagesOne && k + 1 < my_tiles) {
+            if (!two_tiles(k)) {
+                fail_k = k;
+                break;
+            }
+            k += 2;
+        } else {
+            if (!one_tile(k)) {
+                fail_k = k;
+                break;
+            }
+            k += 1;
+        }
     }
 
     if (fail_k >= 0) {
