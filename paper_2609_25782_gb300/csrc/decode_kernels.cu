@@ -185,6 +185,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     // The combine kernel may be scheduled once every CTA of this grid has
     // started; it still waits for this grid to finish before reading.
     asm volatile("griddepcontrol.launch_dependents;");
+    const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
+    // Tables at most 16 x KVT_SPLIT_MIN_TILES tiles wide split every session
+    // every KVT_SPLIT_MIN_TILES tiles, so this warp's tiles are known before
+    // T: their block ids load alongside T instead of after it. Lanes past
+    // the session's tiles may read table entries past its blocks (never used).
+    constexpr int kMinWarpTiles = KVT_SPLIT_MIN_TILES / kDecodeWarps;
+    const bool fixed_split = split_tiles(a.max_blocks * sh.bt) == KVT_SPLIT_MIN_TILES;
+    int early_blk = 0;
+    if (fixed_split && lane < kMinWarpTiles) {
+        const int j = (split * KVT_SPLIT_MIN_TILES + warp + lane * kDecodeWarps) * kTileTokens / sh.bt;
+        if (j < a.max_blocks) early_blk = trow[j];
+    }
     const int T = a.seq_lens[b];
     if (T < 1 || T > a.max_blocks * sh.bt) {
         if (split == 0 && g == 0 && threadIdx.x == 0) atomicOr(a.err, kErrBadLength);
@@ -200,7 +212,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     uint8_t *ring = smem + warp * kStages * kTileBytes;
     const uint32_t ring_s = smem_u32(ring);
     const uint32_t bar0 = smem_u32(bars + warp * kStages);
-    const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
     const int chunk_rows = sh.Hkv * sh.bt;   // rows between K and V runs
 
     // Block ids of this warp's tiles, fetched together up front: lane t
@@ -208,8 +219,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     // of a tile copy (one CTA per SM has no other warps to hide it behind).
     static_assert((KVT_SPLIT_MAX_TILES + kDecodeWarps - 1) / kDecodeWarps <= 32,
                   "a warp's tiles of one split must fit one block id per lane");
-    int lane_blk = 0;
-    if (lane < my_tiles)
+    static_assert(KVT_SPLIT_MIN_TILES % kDecodeWarps == 0, "whole tiles per warp");
+    int lane_blk = early_blk;
+    if (!fixed_split && lane < my_tiles)
         lane_blk = trow[(tile0 + warp + lane * kDecodeWarps) * kTileTokens / sh.bt];
 
     if (lane == 0) {
@@ -598,14 +610,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
 // while K1 drains.
 __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a) {
     asm volatile("griddepcontrol.launch_dependents;");   // a following overlapped call
-    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int64_t row = blockIdx.x;                // lb * Hq + h
     const int lb = static_cast<int>(row / a.s.Hq);
     const int b = lb % a.B;
+    // seq_lens is read before the wait, as K1 reads it: no decode kernel
+    // writes it, so only the partials have to wait for K1 to finish.
     const int T = a.seq_lens[b];
     if (T < 1 || T > a.max_blocks * a.s.bt) return;
     const int ns = num_splits(T);
     if (ns <= 1) return;                           // written by K1
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int64_t base = row * a.max_splits;
