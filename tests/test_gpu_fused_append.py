@@ -162,6 +162,25 @@ def test_fused_steps_cross_blocks_and_splits(pkg):
     pu.close()
 
 
+def test_fused_steps_one_cta_per_sm(pkg):
+    """A batch small enough for one CTA per SM (3 splits x 4 kv-heads x 3
+    sessions = 36 CTAs) runs the kernel whose warps take their tiles in
+    pairs. Over twenty steps the token that arrives with the call lands in
+    the second tile of a pair and in a warp's lone last tile; the fused run
+    stays bit-identical to append-then-decode and agrees with the oracle."""
+    lens = [70, 1100, 2030]
+    pf, sids, T, of, q = run(pkg, True, lens, 20, L=2, mode="layer")
+    pu, _, _, ou, _ = run(pkg, False, lens, 20, L=2, mode="layer")
+    for a, b in zip(of, ou):
+        assert torch.equal(a.view(torch.int32), b.view(torch.int32))
+    check_pool_holds_sessions(pf, sids, T, 2, 16)
+    ref = oracle_out(pf, sids, T, q, 2, 16)
+    assert np.max(np.abs(of[-1].double().numpy() - ref) / np.maximum(1.0, np.abs(ref))) <= TOL
+    assert pf.check_device() == 0
+    pf.close()
+    pu.close()
+
+
 def test_fused_argument_errors(pkg):
     dev = torch.device("cuda:0")
     pool = pkg.Pool(num_layers=1, num_hot_blocks=16, cold_bytes=1 << 20, max_sessions=2,
