@@ -719,6 +719,29 @@ def cpu_baseline(res, seed, budget_s=15.0):
                       f"fp64 CPU oracle, {spent:.1f} s"}
 
 
+def cpu_unpack_baseline(seed, tokens=4096, budget_s=3.0):
+    """The oracle's resume copy timed on the host cores: one session image of
+    `tokens` tokens in the 48-layer shape unpacked into randomly placed hot
+    blocks, repeated while the budget lasts. The copy moves bit patterns, so
+    the values are seeded random bytes."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    nblk = -(-tokens // BT)
+    img = rng.integers(0, 1 << 16, size=(L, 2, HKV, tokens, D), dtype=np.uint16)
+    hot = np.zeros((2 * nblk, L, 2, HKV, BT, D), dtype=np.uint16)
+    row = rng.permutation(2 * nblk)[:nblk].astype(np.int32)
+    spent, reps = 0.0, 0
+    while reps < 1 or spent < budget_s:
+        t0 = time.perf_counter()
+        oracle.unpack(img, tokens, row, hot)
+        spent += time.perf_counter() - t0
+        reps += 1
+    rw = 2 * tokens * TOKEN_BYTES * reps
+    return {"value": round(rw / spent / 1e9, 3), "unit": "GB/s r+w", "cores": 1, "kind": "oracle",
+            "sample": f"unpack of one {tokens}-token image ({tokens * TOKEN_BYTES / 1e9:.2f} GB) "
+                      f"into random blocks, {reps} times, {spent:.1f} s"}
+
+
 METRIC = "decode-attn KV GB/s (per step over all layers; resume-unpack GB/s and ms in secondary)"
 
 
@@ -865,6 +888,8 @@ def main():
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(res, replica_seed(args.seed, rank))
+        if secondary is not None:
+            secondary["resume_unpack"]["cpu_baseline"] = cpu_unpack_baseline(args.seed)
     res["pool"].close()
     del res["pool"]
     torch.cuda.empty_cache()

@@ -105,3 +105,13 @@ def test_traffic_record_goes_null_when_a_source_changes(tmp_path, monkeypatch):
     assert bench.recorded_traffic() is None
     rec.write_text("kernel: k\ndram_bytes_per_launch: 1234\n")   # no hashes: not trusted
     assert bench.recorded_traffic() is None
+
+
+def test_cpu_unpack_baseline_reports_its_sample():
+    """The resume metric's CPU baseline: the oracle's unpack on a bounded,
+    stated sample, with the keys the bench line carries."""
+    sys.path.insert(0, ROOT)
+    import bench
+    r = bench.cpu_unpack_baseline(0, tokens=64, budget_s=0.01)
+    assert r["kind"] == "oracle" and r["cores"] == 1 and r["value"] > 0
+    assert r["unit"] == "GB/s r+w" and "64-token image" in r["sample"]
