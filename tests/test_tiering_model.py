@@ -53,9 +53,9 @@ def test_paper_capacity_figures(tm):
     mean = 0.82 * tm.GIB                       # resident KV per session, steady state
     hbm_only = tm.session_capacity(mean, tm.PAPER_HBM_BYTES)
     tiered = tm.session_capacity(mean, tm.PAPER_HBM_BYTES, cold_tier_bytes=tm.HBF_CAPACITY_BYTES)
-    assert abs(hbm_only - 165) < 1.0           # "saturates at 165 sessions"
-    assert abs(tiered / 3900 - 1) < 0.01       # "expands capacity to 3,900 sessions"
-    assert round(tiered / hbm_only) == 24      # "24x more concurrent sessions"
+    assert abs(hbm_only - 165) < 1.0           # HBM alone: the paper's 165-session limit
+    assert abs(tiered / 3900 - 1) < 0.01       # with the flash tier: its 3,900 sessions
+    assert round(tiered / hbm_only) == 24      # the ratio the paper reports, 24x
     # the cold tier adds to what HBM holds; without the weights' share both would be off
     assert abs(tm.HBF_CAPACITY_BYTES / mean / 3900 - 1) > 0.03
     assert tm.session_capacity(mean, tm.PAPER_HBM_BYTES, weight_bytes=0) > 230
