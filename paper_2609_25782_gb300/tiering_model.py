@@ -2,8 +2,8 @@
 
 * Flash lifetime, Eq. (1) (Section 2, "High bandwidth flash"): the writable
   budget of the cold tier is its capacity C times the rated program/erase
-  cycles N_PE; dividing by the effective write rate R_W * WAF gives the
-  expected service lifetime T_life = C * N_PE / (R_W * WAF).
+  cycles N_PE, and T_life = C * N_PE / (R_W * WAF) is how long that budget
+  lasts at the write rate R_W amplified by the write-amplification factor WAF.
 * Read power (Section 4, "Methodology"): the sum over memory tiers of each
   tier's read rate times its energy per bit. Serving the hot set from flash
   instead of HBM costs (E_flash - E_HBM) * (hot-set read rate) more.
