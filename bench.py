@@ -885,8 +885,8 @@ def main():
         res["pool"] = None
         secondary = run_migration(args, rank)
         res["pool"] = keep
-    cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    cpu = None   # the oracle baselines: rank 0 of a single-GPU run only
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(res, replica_seed(args.seed, rank))
         if secondary is not None:
             secondary["resume_unpack"]["cpu_baseline"] = cpu_unpack_baseline(args.seed)
