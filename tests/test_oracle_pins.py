@@ -62,6 +62,31 @@ def test_paged_matches_dense_bruteforce(bt):
             np.testing.assert_allclose(out[l, b], ref, rtol=1e-10, atol=1e-12)
 
 
+def test_paged_matches_dense_on_drawn_shapes():
+    """The same brute-force pin over drawn shapes: group sizes from MHA to
+    8 q-heads per kv-head, block sizes 1 to 32, head dims 16 to 128, ragged
+    lengths from one token up, and scales including the config-1 reading."""
+    hyp = pytest.importorskip("hypothesis")
+    st = hyp.strategies
+
+    @hyp.settings(max_examples=30, deadline=None, derandomize=True)
+    @hyp.given(hk=st.sampled_from([(4, 4), (8, 2), (8, 1), (6, 3), (32, 4)]),
+               bt=st.sampled_from([1, 4, 16, 32]), D=st.sampled_from([16, 64, 128]),
+               lens=st.lists(st.integers(1, 80), min_size=1, max_size=3),
+               scale=st.sampled_from([1.0, 1 / math.sqrt(128), 0.3]),
+               seed=st.integers(0, 1000))
+    def check(hk, bt, D, lens, scale, seed):
+        Hq, Hkv = hk
+        sess, tables, hot, q = make_case(seed, lens, 1, Hq, Hkv, D, bt)
+        out = oracle.paged_decode(hot, q, tables, lens, scale, Hq)
+        for b, T in enumerate(lens):
+            k, v = synth.session_kv_np(seed, sess[b], [0], Hkv, D, T)
+            ref = dense_attention(q[0, b], k[0], v[0], scale, Hq // Hkv)
+            np.testing.assert_allclose(out[0, b], ref, rtol=1e-10, atol=1e-12)
+
+    check()
+
+
 def test_layer_offset_selects_layer():
     lens = [40, 9]
     sess, tables, hot, q = make_case(3, lens, L=3)
