@@ -235,6 +235,43 @@ def test_pack_unpack_round_trip_and_write_once():
     assert np.array_equal(hot2, hot)
 
 
+def test_migration_copies_on_drawn_shapes():
+    """Unpack against the image reshaped into blocks, pack(unpack(image)) ==
+    image, and a pack from t0 writing exactly tokens [t0, T), over drawn
+    layer counts, kv-head counts, block sizes, lengths and placements."""
+    hyp = pytest.importorskip("hypothesis")
+    st = hyp.strategies
+
+    @hyp.settings(max_examples=30, deadline=None, derandomize=True)
+    @hyp.given(L=st.integers(1, 3), Hkv=st.sampled_from([1, 2, 4]),
+               bt=st.sampled_from([1, 4, 16, 64]), T=st.integers(1, 150),
+               extra=st.integers(0, 40), t0_frac=st.floats(0.0, 1.0),
+               seed=st.integers(0, 1000))
+    def check(L, Hkv, bt, T, extra, t0_frac, seed):
+        D, cap = 16, T + extra
+        img = synth.session_image_np(seed, 3, L, Hkv, D, T, cap, poison_tail=False)
+        nb = -(-T // bt)
+        NB = nb + 3
+        row = synth.random_block_tables(seed, [T], bt, NB)[0]
+        hot = np.zeros((NB, L, 2, Hkv, bt, D), dtype=np.uint16)
+        oracle.unpack(img, T, row, hot)
+        blocks = image_as_blocks(img, T, bt)
+        for j in range(nb):
+            n = min(bt, T - j * bt)
+            assert np.array_equal(hot[row[j], :, :, :, :n], blocks[j][:, :, :, :n])
+        back = np.zeros_like(img)
+        per_tok = oracle.kv_bytes_per_token(L, Hkv, D)
+        assert oracle.pack(hot, row, 0, T, back) == T * per_tok
+        assert np.array_equal(back[:, :, :, :T], img[:, :, :, :T])
+        t0 = int(t0_frac * T)
+        part = np.full_like(img, 0x5A5A)
+        assert oracle.pack(hot, row, t0, T, part) == (T - t0) * per_tok
+        assert np.all(part[:, :, :, :t0] == 0x5A5A) and np.all(part[:, :, :, T:] == 0x5A5A)
+        assert np.array_equal(part[:, :, :, t0:T], img[:, :, :, t0:T])
+
+    check()
+
+
 def test_append_positions():
     L, Hkv, D, bt = 2, 2, 128, 16
     NB = 6
