@@ -48,7 +48,7 @@ def hbm_peak():
         return FALLBACK_HBM, "fallback"
 
 
-TRAFFIC_RECORD = "decode_split_kernel_traffic_48L_B32_8K-32K.txt"
+TRAFFIC_RECORD = "decode_split_kernel_traffic_2L_B32_8K-32K.txt"
 
 
 def recorded_traffic():
@@ -452,7 +452,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     dev = torch.device("cuda", torch.cuda.current_device())
     cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps,
                          admit_lead=args.trace_admit_lead,
-                         fused_append=not args.trace_unfused_append)
+                         fused_append=not args.trace_unfused_append,
+                         prefetch=not args.trace_no_prefetch)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -508,13 +509,66 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     steps_ms = sorted(t for t, _ in step_t)
     # per-step decode bandwidth: separates workload size from interference
     step_gbs = sorted(tok * TOKEN_BYTES / (t * 1e-3) / 1e9 for t, tok in step_t)
-    mig = {"unpack": [0.0, 0], "pack": [0.0, 0]}
+    mig = {"unpack": [0.0, 0], "pack": [0.0, 0], "prefetch": [0.0, 0]}
     for kind, a, b, nbytes in d.mig_events:
         mig[kind][0] += a.elapsed_time(b)
         mig[kind][1] += nbytes
     st = pool.stats()
     pool.close()
     del buf_k, buf_v, flat_k, flat_v
+    # decode/migration overlap (Section 3: eviction and resume run beside
+    # decode): every interval on one device clock, relative to the first step
+    overlap = None
+    if d.step_events and d.mig_events:
+        ref = d.step_events[0][0]
+        steps_iv = [(ref.elapsed_time(a), ref.elapsed_time(b), tok) for a, b, _, tok in d.step_events]
+        migs_iv = [(ref.elapsed_time(a), ref.elapsed_time(b)) for _, a, b, _ in d.mig_events]
+        mig_ms = sum(max(0.0, e - s0) for s0, e in migs_iv)
+        inside = 0.0
+        j = 0
+        for s0, e in sorted(migs_iv):       # steps are disjoint and in time order
+            while j < len(steps_iv) and steps_iv[j][1] <= s0:
+                j += 1
+            i = j
+            while i < len(steps_iv) and steps_iv[i][0] < e:
+                inside += max(0.0, min(e, steps_iv[i][1]) - max(s0, steps_iv[i][0]))
+                i += 1
+        busy, idle = [], []
+        for s0, e, tok in steps_iv:
+            hit = any(ms < e and me > s0 for ms, me in migs_iv)
+            (busy if hit else idle).append(tok * TOKEN_BYTES / max(1e-9, (e - s0) * 1e-3) / 1e9)
+        med = lambda v: round(statistics.median(v), 1) if v else None
+        overlap = {"migration_ms": round(mig_ms, 2),
+                   "migration_overlapping_decode_frac": round(inside / max(1e-9, mig_ms), 4),
+                   "steps_with_migration": len(busy), "steps_without": len(idle),
+                   "decode_kv_gbs_p50_with_migration": med(busy),
+                   "decode_kv_gbs_p50_without": med(idle)}
+    # host side of the run: enqueue time per step, garbage-collector pauses,
+    # and what the host was doing around the slowest step
+    host_ms = sorted((h[3] - h[0]) * 1e3 for h in d.host_stamps)
+    worst = max(range(len(step_t)), key=lambda i: step_t[i][0]) if step_t else None
+    host = {"enqueue_ms_p50": round(host_ms[len(host_ms) // 2], 3),
+            "enqueue_ms_max": round(host_ms[-1], 3),
+            "gc_pauses": len(d.gc_pauses),
+            "gc_pause_ms_max": round(max((p[2] for p in d.gc_pauses), default=0.0) * 1e3, 3)}
+    hk = max(range(len(d.host_stamps)), key=lambda i: d.host_stamps[i][3] - d.host_stamps[i][0])
+    h = d.host_stamps[hk]
+    host["slowest_host_step"] = {
+        "step": hk, "ms": round((h[3] - h[0]) * 1e3, 3),
+        "pauses_admissions_ms": round((h[1] - h[0]) * 1e3, 3),
+        "reserve_ms": round(((h[2] or h[1]) - h[1]) * 1e3, 3),
+        "decode_enqueue_ms": round((h[3] - (h[2] or h[1])) * 1e3, 3),
+        "gpu_ms": round(step_t[d.step_index.index(hk)][0], 3) if hk in d.step_index else None}
+    if worst is not None:
+        k = d.step_index[worst]
+        lo = max(0, k - 8)
+        t_lo, t_hi = d.host_stamps[lo][0], d.host_stamps[k][3]
+        host["slowest_step"] = {
+            "step": k, "ms": round(step_t[worst][0], 3),
+            "host_enqueue_ms": round((d.host_stamps[k][3] - d.host_stamps[k][0]) * 1e3, 3),
+            "host_ms_prev8_max": round(max((h[3] - h[0]) * 1e3 for h in d.host_stamps[lo:k + 1]), 3),
+            "gc_ms_in_prev8": round(sum(p[2] for p in d.gc_pauses
+                                        if t_lo <= p[1] <= t_hi) * 1e3, 3)}
     torch.cuda.empty_cache()
 
     def pct(p):
@@ -540,16 +594,22 @@ def run_trace(args, rank, lru_factor: float = 0.0):
                  "blocks_evicted": st["blocks_evicted"],
                  "cold_write_gb": round(st["bytes_packed"] / 1e9, 2),
                  "cold_read_gb": round(st["bytes_unpacked"] / 1e9, 2),
+                 "prefetch": cfg.prefetch,
+                 "blocks_prefetched": st["blocks_prefetched"],
+                 "blocks_fetched_in_step": st["batch_blocks_fetched"],
+                 "prefetch_skipped": d.counts["prefetch_skipped"],
                  "matches_dry_run": all(st[k] == dry[k] for k in (
                      "bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
-                     "resume_blocks_missed", "resumes", "pauses"))})
+                     "resume_blocks_missed", "resumes", "pauses", "batch_blocks_fetched",
+                     "blocks_prefetched", "prefetches"))})
     return {
         **extra,
         "admit_lead": cfg.admit_lead, "mig_ctas": args.trace_mig_ctas,
         "step_append": "fused into the decode kernel" if cfg.fused_append else "separate kernel",
         "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
         "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
-        "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2),
+        "step_ms_max": round(steps_ms[-1], 3), "wall_s": round(wall, 2), "host": host,
+        "overlap": overlap,
         "mean_batch": round(sum(e[2] for e in d.step_events) / max(1, len(d.step_events)), 2),
         "step_kv_gbs_p50": round(step_gbs[len(step_gbs) // 2], 1),
         "step_kv_gbs_p1": round(step_gbs[len(step_gbs) // 100], 1),
@@ -821,6 +881,10 @@ def main():
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--only-trace", action="store_true",
                     help="run only the agentic trace (simple and residency modes)")
+    ap.add_argument("--trace-no-prefetch", action="store_true",
+                    help="trace (residency mode): no one-step-ahead fetch of spilled blocks")
+    ap.add_argument("--trace-lru-factor", type=float, default=1.5,
+                    help="residency-mode hot pool as a multiple of the simple mode's peak")
     ap.add_argument("--trace-unfused-append", action="store_true",
                     help="trace: write each step's token with its own kernel before the decode")
     ap.add_argument("--no-trace", action="store_true")
@@ -862,7 +926,7 @@ def main():
         return 0
     if args.only_trace:
         tr_res = {"trace": run_trace(args, rank),
-                  "trace_lru": run_trace(args, rank, lru_factor=1.5)}
+                  "trace_lru": run_trace(args, rank, lru_factor=args.trace_lru_factor)}
         if rank == 0:
             print(json.dumps(tr_res))
         return 0
@@ -895,7 +959,7 @@ def main():
     torch.cuda.empty_cache()
     if secondary is not None and not args.no_trace:
         secondary["trace"] = run_trace(args, rank)
-        secondary["trace_lru"] = run_trace(args, rank, lru_factor=1.5)
+        secondary["trace_lru"] = run_trace(args, rank, lru_factor=args.trace_lru_factor)
     nl, nbatch = args.layers, args.batch
     headline = (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2)
 

@@ -133,15 +133,29 @@ typedef struct kv_pool_stats {
     int64_t blocks_evicted;       /* residency mode: blocks evicted            */
     int64_t resume_blocks_hit;    /* residency mode: still hot at resume       */
     int64_t resume_blocks_missed; /* residency mode: fetched at resume         */
+    int64_t batch_blocks_fetched; /* residency mode: fetched by kv_pool_batch_tables
+                                   * or kv_pool_batch_reserve (inside a step)  */
+    int64_t blocks_prefetched;    /* residency mode: fetched by kv_pool_prefetch */
+    int64_t prefetches;           /* kv_pool_prefetch calls that did their work */
 } kv_pool_stats;
 
-/* Create a pool over caller-owned arenas. The hot free list starts as
- * 0..num_hot_blocks-1 shuffled by Fisher-Yates driven by splitmix64 seeded
- * with alloc_seed (draw j = floor(r * (i+1) / 2^64) for i = n-1 .. 1);
- * allocations pop from its end. *out receives the pool. */
+/* Create a pool over caller-owned arenas. Bookkeeping; no passage of the
+ * paper defines pool set-up. What it sets up does have one: the hot pool of
+ * fixed-size paged blocks (Section 2, "Large Language Models"; one block =
+ * 16 tokens of every layer, the 1.5 MiB unit of Section 4, "Methodology")
+ * and the cold pool of per-session images (Section 3, "Architecture and
+ * data paths"). The hot free list starts as 0..num_hot_blocks-1 shuffled by
+ * Fisher-Yates driven by splitmix64 seeded with alloc_seed (draw
+ * j = floor(r * (i+1) / 2^64) for i = n-1 .. 1); allocations pop from its
+ * end. Allocates the pool's device metadata (tables, decode workspace, flag
+ * word) with cudaMalloc. *out receives the pool. Errors: bad shape or null
+ * or misaligned arenas -> KV_ERR_INVALID_ARG; a failing CUDA call ->
+ * KV_ERR_CUDA (nothing is left allocated). */
 int kv_pool_create(const kv_pool_config *cfg, kv_pool **out);
 
-/* Destroy a pool after synchronising its device. Arenas are not freed. */
+/* Destroy a pool after synchronising its device. Bookkeeping; no passage.
+ * Frees the pool's own device metadata and events; the caller's arenas are
+ * not freed. */
 int kv_pool_destroy(kv_pool *pool);
 
 /* Bytes of one hot block: L * 2 * Hkv * bt * D * 2. */
@@ -159,9 +173,13 @@ int64_t kv_token_bytes(const kv_pool_config *cfg);
 int32_t kv_decode_splits(int64_t t);
 
 /* Create an ACTIVE, empty session able to hold max_tokens (1 ..
- * max_context) tokens; reserves its cold image (max_tokens * token bytes)
- * in the cold arena (first fit). Errors: KV_ERR_NO_COLD_SPACE, too many
- * sessions -> KV_ERR_INVALID_ARG. */
+ * max_context) tokens. Bookkeeping; no passage defines the call. A session
+ * is the paper's unit of agentic serving, whose context keeps growing
+ * across turns (Section 2, "Agentic AI Serving"); its cold image is the
+ * per-session region that data path 4 writes (Section 3). Reserves the
+ * image (max_tokens * token bytes, rounded up to 256 B) in the cold arena
+ * (first fit). Errors: KV_ERR_NO_COLD_SPACE, too many sessions ->
+ * KV_ERR_INVALID_ARG. */
 int session_create(kv_pool *pool, int64_t max_tokens, int32_t *sid_out);
 
 /* Create a PAUSED session whose image the caller fills with `tokens` valid
@@ -265,16 +283,38 @@ int session_pause(kv_pool *pool, int32_t sid, kv_stream_t stream);
 int session_resume(kv_pool *pool, int32_t sid, kv_stream_t stream);
 
 /* Event recorded after the session's last resume (NULL if none): a decode
- * stream waits on it before reading the session's blocks. */
+ * stream waits on it before reading the session's blocks (Section 3,
+ * "Eviction, resume and decode": a resumed session decodes once its KV is
+ * back in HBM; resume overlaps other work). The event is owned by the pool
+ * and stays valid until the session is destroyed. */
 int session_ready_event(kv_pool *pool, int32_t sid, kv_event_t *ev);
 
 /* State, length, capacity, cold_valid and image address of a session. */
 int session_info(kv_pool *pool, int32_t sid, kv_session_info *out);
 
 /* Host copy of a session's block-table row: up to cap entries into
- * host_row; *nblocks receives the row length. */
+ * host_row; *nblocks receives the row length. Bookkeeping; no passage (the
+ * table maps a session's logical blocks to the fixed-size paged blocks of
+ * Section 2, "Large Language Models"). Residency mode: an evicted block's
+ * entry is -1. */
 int session_block_table(kv_pool *pool, int32_t sid, int32_t *host_row, int32_t cap,
                         int32_t *nblocks);
+
+/* Device address of a session's block-table row in the pool's table arena
+ * (int32, at least ceil(max_context / block_tokens) entries; *nblocks
+ * receives the number of logical blocks). Bookkeeping; no passage. For
+ * callers that form their own decode batch tables on the device instead of
+ * calling kv_pool_batch_tables. The pool owns the memory; the address stays
+ * fixed for the pool's life. The row's entries are written by kernels on
+ * the stream of the call that changed them (append, resume,
+ * kv_pool_batch_reserve, a residency-mode fetch): read it on a stream
+ * ordered after that call. Residency mode: the entry of a block that was
+ * evicted is stale (it names a slot that may hold another session's block)
+ * until the block is fetched back; use the row only while session_info
+ * reports num_blocks == ceil(tokens / block_tokens). Host-logic-only pools
+ * have no device arena: KV_ERR_BAD_STATE. */
+int session_block_table_device(kv_pool *pool, int32_t sid, const int32_t **dev_row,
+                               int32_t *nblocks);
 
 /* Build the decode inputs of a batch of ACTIVE sessions: block_tables
  * (device int32 [B][max_blocks], entries past a row's length set to -1) and
@@ -302,6 +342,30 @@ int kv_pool_batch_tables(kv_pool *pool, const int32_t *sids, int32_t B, int32_t 
 int kv_pool_batch_reserve(kv_pool *pool, const int32_t *sids, int32_t B, int32_t *block_tables,
                           int32_t max_blocks, int32_t *seq_lens, kv_stream_t stream);
 
+/* Prefetch one step ahead of decode (Section 3, "Eviction, resume and
+ * decode": decode reads a known set of blocks each step, so the next step's
+ * blocks are fetched ahead and flash latency stays off the step). sids: host
+ * array of the B ACTIVE sessions of the NEXT decode step; busy: host array of
+ * the n_busy sessions whose decode may still be running (the current step's
+ * batch), or NULL with n_busy = 0. In residency mode every evicted block of
+ * the next batch is fetched on `stream` (typically a migration stream, so it
+ * runs beside the current step), victims coming only from sessions in
+ * neither array (LRU order as for any allocation, written on eviction only
+ * for tokens the image lacks); the next batch's sessions are then stamped
+ * with one recency time, and each session that had blocks fetched
+ * re-records its ready event on `stream`, which kv_pool_batch_reserve and
+ * kv_pool_batch_tables wait on before the step reads them. The stream must
+ * already be ordered after the decode steps before the current one (they
+ * may have read or written the victims). Pops from the free list go member
+ * by member, missing blocks in ascending order. Simple mode: nothing is ever
+ * evicted, the call only validates and returns KV_OK. Errors: unknown or
+ * paused session -> KV_ERR_INVALID_ARG / KV_ERR_BAD_STATE; not enough
+ * evictable blocks outside both arrays -> KV_ERR_NO_HOT_BLOCKS (nothing
+ * changes; the step's own batch call will then fetch what is missing, with
+ * victims outside the next batch only). All or nothing. */
+int kv_pool_prefetch(kv_pool *pool, const int32_t *sids, int32_t B, const int32_t *busy,
+                     int32_t n_busy, kv_stream_t stream);
+
 /* Re-run the Fisher-Yates shuffle over the current free list with a new
  * seed (scrambles where the next allocations land). */
 int kv_pool_shuffle_free(kv_pool *pool, uint64_t seed);
@@ -326,7 +390,7 @@ int kv_pool_check_device(kv_pool *pool, int32_t *flags);
 /* Cap the migration kernels (resume-unpack, pause-pack, evictions) at
  * max_ctas CTAs of 256 threads, so that migrations running beside decode take
  * a smaller share of HBM bandwidth (Section 3, data paths: eviction and resume
- * overlap decode). 0 removes the cap (the default grid: 16 CTAs per SM).
+ * overlap decode). 0 removes the cap (the default grid: 32 CTAs per SM).
  * Affects later calls only. */
 int kv_pool_set_migration_limit(kv_pool *pool, int32_t max_ctas);
 
@@ -375,12 +439,20 @@ int kv_pool_inject_decode_timeout(kv_pool *pool, int32_t on);
  * capture. All calls share the one array: calls whose work overlaps on the
  * GPU (different streams, or different host threads without ordering) race
  * and give wrong results; order them on one stream. Kernel bounds checks
- * keep bad block ids or lengths memory-safe but are not reported here. */
+ * keep bad block ids or lengths memory-safe but are not reported here: a
+ * row whose seq_len is below 1 or beyond max_blocks * block_tokens is not
+ * written at all (out keeps what it held), a block id outside the pool is
+ * read as block 0 (that row's output is then wrong), and a tile wait that
+ * runs out (2 s) leaves that row's output undefined. The tensor map of a
+ * hot arena is encoded on its first call and kept (host memory, four
+ * arenas per device). */
 int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer, const void *q,
                              const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                              int32_t max_blocks, float scale, float *out, kv_stream_t stream);
 
-/* Message of the last error on the calling thread ("" if none). */
+/* Message of the last error on the calling thread ("" if none).
+ * Bookkeeping; no passage. The string is owned by the library and valid
+ * until the thread's next failing call. */
 const char *kv_last_error(void);
 
 #ifdef __cplusplus

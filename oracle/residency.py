@@ -54,7 +54,8 @@ class ResidencyOracle:
         self.clock = 0
         self.s: dict[int, Sess] = {}
         self.stats = {"bytes_packed": 0, "bytes_unpacked": 0, "bytes_appended": 0,
-                      "blocks_evicted": 0, "resume_blocks_hit": 0, "resume_blocks_missed": 0}
+                      "blocks_evicted": 0, "resume_blocks_hit": 0, "resume_blocks_missed": 0,
+                      "batch_blocks_fetched": 0, "blocks_prefetched": 0, "prefetches": 0}
         self.log = []              # ("pack"|"unpack", sid, j, slot, t0, t1) in issue order
 
     # ----------------------------------------------------------- helpers
@@ -152,17 +153,36 @@ class ResidencyOracle:
         s.state = "active"
         s.time = self._tick()
 
-    def batch(self, sids: list):
-        need = [(sid, [j for j, slot in enumerate(self.s[sid].slots) if slot < 0]) for sid in sids]
+    def _bring_back(self, sids: list, protect: set) -> int:
+        """Fetch every missing block of `sids` (each session once, in order of
+        first appearance), evicting outside `protect`; stamp them all with one
+        time. Returns the number of blocks fetched."""
+        uniq = list(dict.fromkeys(sids))
+        need = [(sid, [j for j, slot in enumerate(self.s[sid].slots) if slot < 0]) for sid in uniq]
         total = sum(len(m) for _, m in need)
-        self._check_room(total, set(sids))
-        self._evict(total, set(sids))
+        self._check_room(total, protect)
+        self._evict(total, protect)
         for sid, missing in need:
             if missing:
                 self._fetch(sid, missing)
         t = self._tick()
-        for sid in sids:
+        for sid in uniq:
             self.s[sid].time = t
+        return total
+
+    def batch(self, sids: list):
+        self.stats["batch_blocks_fetched"] += self._bring_back(sids, set(sids))
+
+    def prefetch(self, sids: list, busy: list = ()):
+        """One step ahead of decode (Section 3, "Eviction, resume and
+        decode"): the next step's sessions get their evicted blocks back now,
+        while the current step (the sessions in `busy`) is still decoding, so
+        victims may belong to neither. All or nothing; the next step's
+        sessions are stamped as used."""
+        for sid in sids:
+            assert self.s[sid].state == "active"
+        self.stats["blocks_prefetched"] += self._bring_back(sids, set(sids) | set(busy))
+        self.stats["prefetches"] += 1
 
     def batch_reserve(self, sids: list):
         """One decode step's fresh token for each session of the batch (its
@@ -184,6 +204,7 @@ class ResidencyOracle:
             s = self.s[sid]
             if missing:
                 self._fetch(sid, missing)
+                self.stats["batch_blocks_fetched"] += len(missing)
             if grow:
                 s.slots.append(int(self.fl.pop(1)[0]))
                 s.img.append(0)

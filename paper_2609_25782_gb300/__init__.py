@@ -109,6 +109,15 @@ class Pool:
         kvtier.kv_pool_batch_reserve(self.handle, list(sids), block_tables, max_blocks, seq_lens,
                                      stream)
 
+    def prefetch(self, next_sids, busy=(), stream=None) -> None:
+        """Fetch the next step's evicted blocks ahead of it (residency mode),
+        victims outside next_sids and busy (the step still being decoded)."""
+        kvtier.kv_pool_prefetch(self.handle, list(next_sids), list(busy), stream)
+
+    def session_block_table_device(self, sid: int) -> tuple[int, int]:
+        """(device address of the session's table row, logical blocks)."""
+        return kvtier.session_block_table_device(self.handle, sid)
+
     def decode_attention(self, layer: int, q, block_tables, seq_lens, B: int, max_blocks: int,
                          scale: float, out, stream=None, overlap_previous: bool = False) -> None:
         """out: fp32, or bf16 (then the result is rounded to nearest even)."""

@@ -682,13 +682,15 @@ static int lru_resume(kv_pool *p, int32_t sid, cudaStream_t st) {
     return KV_OK;
 }
 
-// Before a decode step: bring back any block of the batch's sessions that was
-// evicted (no pinning: under pressure even active blocks spill), then stamp
-// all of them with one new recency time.
-static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStream_t st) {
-    std::vector<int32_t> uniq;
-    for (int32_t i = 0; i < B; ++i)
-        if (std::find(uniq.begin(), uniq.end(), sids[i]) == uniq.end()) uniq.push_back(sids[i]);
+// Bring back every evicted block of the sessions `uniq` (no pinning: under
+// pressure even active blocks spill), with victims from sessions outside
+// `protect`, then stamp all of `uniq` with one new recency time. With
+// record_ready, each session that had a block fetched re-records its ready
+// event on `st` (a decode stream waits on it). *blocks receives the number
+// of blocks fetched.
+static int lru_fetch(kv_pool *p, const std::vector<int32_t> &uniq,
+                     const std::vector<int32_t> &protect, bool record_ready, cudaStream_t st,
+                     int64_t *blocks) {
     std::vector<std::vector<int32_t>> miss(uniq.size());
     int64_t need = 0;
     for (size_t u = 0; u < uniq.size(); ++u) {
@@ -698,7 +700,7 @@ static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStrea
         need += static_cast<int64_t>(miss[u].size());
     }
     std::vector<Victim> vic;
-    if (!p->plan_evict(need, uniq, vic))
+    if (!p->plan_evict(need, protect, vic))
         return fail(KV_ERR_NO_HOT_BLOCKS, "the batch's blocks do not fit in the hot pool");
     const std::vector<int32_t> got = p->peek_alloc(need, vic);
     std::vector<std::vector<int32_t>> rows(uniq.size());
@@ -714,8 +716,16 @@ static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStrea
             ++k;
         }
     }
-    int rc = p->evict_device(vic, st);
+    int rc = KV_OK;
+    for (size_t u = 0; !rc && record_ready && u < uniq.size(); ++u)
+        if (!miss[u].empty()) rc = ensure_event(p, &p->sessions[uniq[u]].ready);
+    if (!rc) rc = p->evict_device(vic, st);
     if (!rc) rc = p->run_jobs(jobs, false, st);   // the fetches also write their table entries
+    for (size_t u = 0; !rc && record_ready && !p->host_only && u < uniq.size(); ++u)
+        if (!miss[u].empty()) {
+            cudaEvent_t ev = p->sessions[uniq[u]].ready;
+            rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(ev, st); });
+        }
     if (rc) return rc;
 
     p->evict_commit(vic);
@@ -728,11 +738,30 @@ static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStrea
         s.hot_count += static_cast<int64_t>(miss[u].size());
         s.last_use = stamp;
         p->lru_in(uniq[u]);
+        if (record_ready && !miss[u].empty()) s.ready_recorded = !p->host_only;
     }
     p->stats.free_blocks -= need;
     p->stats.used_blocks += need;
     p->stats.bytes_unpacked += fetched * p->token_bytes;
+    *blocks = need;
     return KV_OK;
+}
+
+static std::vector<int32_t> unique_ids(const int32_t *ids, int32_t n) {
+    std::vector<int32_t> u;
+    for (int32_t i = 0; i < n; ++i)
+        if (std::find(u.begin(), u.end(), ids[i]) == u.end()) u.push_back(ids[i]);
+    return u;
+}
+
+// Before a decode step: the batch's evicted blocks come back on the step's
+// own stream; victims are outside the batch.
+static int lru_fetch_batch(kv_pool *p, const int32_t *sids, int32_t B, cudaStream_t st) {
+    const std::vector<int32_t> uniq = unique_ids(sids, B);
+    int64_t blocks = 0;
+    int rc = lru_fetch(p, uniq, uniq, false, st, &blocks);
+    if (!rc) p->stats.batch_blocks_fetched += blocks;
+    return rc;
 }
 
 int session_append(kv_pool *p, int32_t sid, const void *k, const void *v, int32_t n,
@@ -1018,6 +1047,17 @@ int session_block_table(kv_pool *p, int32_t sid, int32_t *host_row, int32_t cap,
     return KV_OK;
 }
 
+int session_block_table_device(kv_pool *p, int32_t sid, const int32_t **dev_row,
+                               int32_t *nblocks) {
+    if (!p || !dev_row || !nblocks) return fail(KV_ERR_INVALID_ARG, "null argument");
+    Session *s = p->session(sid);
+    if (!s) return fail(KV_ERR_INVALID_ARG, "no such session");
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "host-logic-only pools have no device tables");
+    *dev_row = p->d_tables + static_cast<int64_t>(sid) * p->table_stride;
+    *nblocks = static_cast<int32_t>(s->blocks.size());
+    return KV_OK;
+}
+
 // Device inputs of a decode batch from the pool's tables: row b of
 // block_tables (entries past the session's length set to -1) and seq_lens.
 // lens / nblk / new_blk, when given, replace the sessions' current lengths
@@ -1176,8 +1216,40 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
     p->stats.free_blocks -= need;
     p->stats.used_blocks += need;
     p->stats.bytes_unpacked += fetched * p->token_bytes;
+    p->stats.batch_blocks_fetched += static_cast<int64_t>(jobs.size());
     p->stats.bytes_appended += static_cast<int64_t>(B) * p->token_bytes;
     p->stats.appends += B;
+    return KV_OK;
+}
+
+// One step ahead of decode (Section 3, "Eviction, resume and decode": decode
+// reads a known set of blocks, so the next step's can be fetched while the
+// current step runs). Victims come from sessions in neither the next batch
+// nor `busy`, the batch the current step is still reading.
+int kv_pool_prefetch(kv_pool *p, const int32_t *sids, int32_t B, const int32_t *busy,
+                     int32_t n_busy, kv_stream_t stream_) {
+    if (!p || !sids || B < 1 || n_busy < 0 || (n_busy > 0 && !busy))
+        return fail(KV_ERR_INVALID_ARG, "bad argument");
+    for (int32_t i = 0; i < B; ++i) {
+        Session *s = p->session(sids[i]);
+        if (!s) return fail(KV_ERR_INVALID_ARG, "no such session in the next batch");
+        if (s->state != KV_SESSION_ACTIVE)
+            return fail(KV_ERR_BAD_STATE, "paused session in the next batch");
+    }
+    for (int32_t i = 0; i < n_busy; ++i)
+        if (!p->session(busy[i])) return fail(KV_ERR_INVALID_ARG, "no such session in busy");
+    if (!p->lru) return KV_OK;   // simple mode: an active session's blocks are always hot
+    const std::vector<int32_t> uniq = unique_ids(sids, B);
+    std::vector<int32_t> protect(uniq);
+    for (int32_t i = 0; i < n_busy; ++i)
+        if (std::find(protect.begin(), protect.end(), busy[i]) == protect.end())
+            protect.push_back(busy[i]);
+    DeviceGuard dg(p->cfg.device, !p->host_only);
+    int64_t blocks = 0;
+    int rc = lru_fetch(p, uniq, protect, true, reinterpret_cast<cudaStream_t>(stream_), &blocks);
+    if (rc) return rc;
+    p->stats.blocks_prefetched += blocks;
+    p->stats.prefetches += 1;
     return KV_OK;
 }
 

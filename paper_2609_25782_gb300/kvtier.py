@@ -39,6 +39,7 @@ EXPORTS = [
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
     "decode_attention_ex", "kv_pool_set_migration_limit", "kv_pool_batch_reserve",
     "decode_append_attention", "kv_pool_inject_decode_timeout", "kv_decode_splits",
+    "session_block_table_device", "kv_pool_prefetch",
 ]
 
 KV_DEVICE_BAD_BLOCK, KV_DEVICE_BAD_LENGTH, KV_DEVICE_TIMEOUT = 1, 2, 4
@@ -71,7 +72,8 @@ class kv_pool_stats(C.Structure):
     _fields_ = [(n, C.c_int64) for n in (
         "free_blocks", "used_blocks", "cold_bytes_used", "bytes_unpacked", "bytes_packed",
         "bytes_appended", "resumes", "pauses", "appends", "decodes", "blocks_evicted",
-        "resume_blocks_hit", "resume_blocks_missed")]
+        "resume_blocks_hit", "resume_blocks_missed", "batch_blocks_fetched",
+        "blocks_prefetched", "prefetches")]
 
 
 class KVError(RuntimeError):
@@ -97,6 +99,7 @@ def _load():
         "session_destroy": [p, i32],
         "session_append": [p, i32, p, p, i32, p],
         "kv_pool_batch_reserve": [p, p, i32, p, i32, p, p],
+        "kv_pool_prefetch": [p, p, i32, p, i32, p],
         "decode_append_attention": [p, i32, p, p, p, p, p, i32, i32, C.c_float, p, C.c_uint32, p],
         "decode_attention": [p, i32, p, p, p, i32, i32, C.c_float, p, p],
         "decode_attention_ex": [p, i32, p, p, p, i32, i32, C.c_float, p, C.c_uint32, p],
@@ -105,6 +108,7 @@ def _load():
         "session_ready_event": [p, i32, C.POINTER(p)],
         "session_info": [p, i32, C.POINTER(kv_session_info)],
         "session_block_table": [p, i32, p, i32, C.POINTER(i32)],
+        "session_block_table_device": [p, i32, C.POINTER(p), C.POINTER(i32)],
         "kv_pool_batch_tables": [p, p, i32, p, i32, p, p],
         "kv_pool_shuffle_free": [p, u64],
         "kv_pool_free_list": [p, p, i64, C.POINTER(i64)],
@@ -256,6 +260,14 @@ def session_block_table(pool: int, sid: int) -> list[int]:
     return list(buf[: n.value])
 
 
+def session_block_table_device(pool: int, sid: int) -> tuple[int, int]:
+    """(device address of the session's table row, number of logical blocks)."""
+    row, n = C.c_void_p(), C.c_int32()
+    _check(lib.session_block_table_device(pool, sid, C.byref(row), C.byref(n)),
+           "session_block_table_device")
+    return row.value, n.value
+
+
 def kv_pool_batch_tables(pool: int, sids, block_tables, max_blocks: int, seq_lens,
                          stream=None) -> None:
     arr = (C.c_int32 * len(sids))(*sids)
@@ -268,6 +280,13 @@ def kv_pool_batch_reserve(pool: int, sids, block_tables, max_blocks: int, seq_le
     arr = (C.c_int32 * len(sids))(*sids)
     _check(lib.kv_pool_batch_reserve(pool, arr, len(sids), _addr(block_tables), max_blocks,
                                      _addr(seq_lens), _stream(stream)), "kv_pool_batch_reserve")
+
+
+def kv_pool_prefetch(pool: int, sids, busy=(), stream=None) -> None:
+    arr = (C.c_int32 * len(sids))(*sids)
+    barr = (C.c_int32 * len(busy))(*busy) if len(busy) else None
+    _check(lib.kv_pool_prefetch(pool, arr, len(sids), barr, len(busy), _stream(stream)),
+           "kv_pool_prefetch")
 
 
 def kv_pool_shuffle_free(pool: int, seed: int) -> None:

@@ -21,8 +21,10 @@ decides what to call and when.
 from __future__ import annotations
 
 import dataclasses
+import gc
 import heapq
 import math
+import time
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -51,6 +53,7 @@ class TraceConfig:
     lru: bool = False                # block residency with LRU write-on-evict
     admit_lead: int = 1              # steps between a resume and the session's first decode
     fused_append: bool = True        # step token written by the decode kernel itself
+    prefetch: bool = True            # residency mode: next step's spilled blocks fetched ahead
 
 
 @dataclass
@@ -113,10 +116,15 @@ class TraceDriver:
         self.peak_tokens = list(self.tokens)
         self.peak_blocks = 0
         self.counts = {"resumes": 0, "pauses": 0, "appended_tokens": 0, "decode_tokens": 0,
-                       "turn_tokens": 0, "steps": 0,
+                       "turn_tokens": 0, "steps": 0, "prefetch_skipped": 0,
                        "session_tokens": 0}   # sum over steps of all sessions' lengths
-        self.step_events = []                # (start, end) per step (gpu)
+        self.step_events = []                # (start, end, B, tokens) per decode step (gpu)
+        self.step_index = []                 # trace step k of each step_events entry
         self.mig_events = []                 # (kind, start, end, bytes)
+        # host clock (perf_counter) per trace step: begin, after pauses and
+        # admissions, after the batch reservation, end of enqueue
+        self.host_stamps = []
+        self.gc_pauses = []                  # (generation, start, seconds) during run()
         self.admit_ev = {}
         self.last_decode_ev = None
         if gpu:
@@ -165,6 +173,8 @@ class TraceDriver:
     # ------------------------------------------------------------------- step
     def step(self, k: int) -> None:
         cfg = self.cfg
+        h0 = time.perf_counter()
+        h_adm = h_res = None
         now = k * cfg.dt_s
         tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
         # 1. sessions whose burst ended last step pause. Simple mode packs their
@@ -210,6 +220,7 @@ class TraceDriver:
             self.joining.append((k + max(1, cfg.admit_lead), i))
             self.counts["resumes"] += 1
         # 3. decode step for the active batch
+        h_adm = time.perf_counter()
         members = sorted(self.active)
         if members:
             if self.gpu:
@@ -243,6 +254,7 @@ class TraceDriver:
                 if self.gpu:
                     kvtier.kv_pool_batch_tables(self.pool, sids, self.tables, mb,
                                                 self.seq_lens, self.dstream)
+            h_res = time.perf_counter()
             self.counts["appended_tokens"] += len(members)
             blocks = sum(-(-self.tokens[i] // cfg.block_tokens)
                          for i in self.active + [i for _, i in self.joining])
@@ -265,6 +277,7 @@ class TraceDriver:
                 end.record(self.dstream)
                 self.last_decode_ev = end
                 self.step_events.append((start, end, B, sum(self.tokens[i] for i in members)))
+                self.step_index.append(k)
                 if self.on_step is not None:
                     self.on_step(k, members)
             self.counts["decode_tokens"] += sum(self.tokens[i] for i in members)
@@ -272,12 +285,63 @@ class TraceDriver:
                 self.burst_left[i] -= 1
                 if self.burst_left[i] <= 0:
                     self.retire.append(i)
+            if cfg.lru and cfg.prefetch:
+                self._prefetch_next(k, sids)
         self.counts["steps"] += 1
         self.counts["session_tokens"] += sum(self.tokens)
+        self.host_stamps.append((h0, h_adm, h_res, time.perf_counter()))
+
+    def _prefetch_next(self, k: int, busy: list) -> None:
+        """One step ahead (Section 3, "Eviction, resume and decode"): the
+        sessions of step k+1 are known now (this step's members minus those
+        whose burst just ended, plus the admitted sessions that join at k+1),
+        so their evicted blocks are fetched on the migration stream while
+        step k decodes; victims exclude both batches. The migration stream is
+        already ordered after step k-1's decode (start of this step)."""
+        retiring = set(self.retire)
+        nxt = sorted({i for i in self.active if i not in retiring} |
+                     {i for j, i in self.joining if j <= k + 1})
+        if not nxt:
+            return
+        sids = [self.sids[i] for i in nxt]
+
+        def call():
+            try:
+                kvtier.kv_pool_prefetch(self.pool, sids, busy, self.mstream if self.gpu else None)
+            except kvtier.KVError as e:   # too few victims outside both batches: the
+                if e.code != kvtier.KV_ERR_NO_HOT_BLOCKS:   # step's own call fetches them
+                    raise
+                self.counts["prefetch_skipped"] += 1
+
+        if self.gpu:
+            before = kvtier.kv_pool_get_stats(self.pool)["blocks_prefetched"]
+            self._record_mig("prefetch", call, 0)
+            n = kvtier.kv_pool_get_stats(self.pool)["blocks_prefetched"] - before
+            kind, a, b, _ = self.mig_events[-1]
+            tok_bytes = self.cfg.layers * 2 * self.cfg.num_kv_heads * 128 * 2
+            self.mig_events[-1] = (kind, a, b, n * self.cfg.block_tokens * tok_bytes)
+        else:
+            call()
 
     def run(self, steps: int | None = None) -> None:
-        for k in range(self.cfg.steps if steps is None else steps):
-            self.step(k)
+        """Run the schedule; Python garbage-collector pauses that fall inside
+        it are recorded in gc_pauses (a host stall long enough to drain the
+        launch queue shows up as a longer step)."""
+        started = {}
+
+        def on_gc(phase, info):
+            if phase == "start":
+                started["t"] = time.perf_counter()
+            elif "t" in started:
+                t = started.pop("t")
+                self.gc_pauses.append((info.get("generation", -1), t, time.perf_counter() - t))
+
+        gc.callbacks.append(on_gc)
+        try:
+            for k in range(self.cfg.steps if steps is None else steps):
+                self.step(k)
+        finally:
+            gc.callbacks.remove(on_gc)
 
 
 def plan(cfg: TraceConfig, trace: list[SessionTrace], hot_blocks: int | None = None) -> dict:

@@ -98,6 +98,12 @@ int main(void) {
                 KV_ERR_INVALID_ARG);
     expect_code("append past capacity", session_append(pool, s1, NULL, NULL, 500, NULL),
                 KV_ERR_INVALID_ARG);
+    {
+        const int32_t *dev_row = NULL;
+        int32_t nb = 0;
+        expect_code("device table row on a host-logic pool",
+                    session_block_table_device(pool, s0, &dev_row, &nb), KV_ERR_BAD_STATE);
+    }
     batch[1] = s0;
     expect_code("session twice in a batch",
                 kv_pool_batch_reserve(pool, batch, 2, NULL, 64, NULL, NULL), KV_ERR_INVALID_ARG);

@@ -205,7 +205,7 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
     pool, tb = lib_pool(kv, nb, seed)
     o = ResidencyOracle(nb, BT, seed=seed, token_bytes=tb)
     live = []
-    fails = reserved = 0
+    fails = reserved = prefetched = 0
     for step in range(500):
         r = rnd.random()
         try:
@@ -276,6 +276,24 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
                     except kv.KVError as e:
                         assert e.code == exp
                         fails += 1
+                elif r < 0.92:      # the next step's blocks, ahead of it
+                    act = [x for x in live if o.s[x].state == "active"]
+                    if not act:
+                        continue
+                    nxt = rnd.sample(act, k=min(len(act), rnd.randint(1, 3)))
+                    busy = rnd.sample(act, k=min(len(act), rnd.randint(0, 2)))
+                    exp = None
+                    try:
+                        o.prefetch(nxt, busy)
+                    except NoHotBlocks:
+                        exp = kv.KV_ERR_NO_HOT_BLOCKS
+                    try:
+                        kv.kv_pool_prefetch(pool, nxt, busy)
+                        assert exp is None
+                        prefetched += 1
+                    except kv.KVError as e:
+                        assert e.code == exp
+                        fails += 1
                 else:               # a fused decode step's token for each member
                     batch = [x for x in live if o.s[x].state == "active" and o.s[x].T < 400]
                     batch = rnd.sample(batch, k=min(len(batch), rnd.randint(1, 3)))
@@ -298,6 +316,7 @@ def test_library_matches_oracle_on_random_sequences(kv, seed):
         compare(kv, pool, o, live)
     st = kv.kv_pool_get_stats(pool)
     assert st["blocks_evicted"] > 20 and st["resume_blocks_missed"] > 0 and reserved > 10
+    assert prefetched > 5 and st["blocks_prefetched"] > 0
     kv.kv_pool_destroy(pool)
 
 
@@ -344,3 +363,79 @@ def test_batch_reserve_simple_mode_equals_one_token_appends(kv):
                       kv.session_info(a, 0).tokens)
     kv.kv_pool_destroy(a)
     kv.kv_pool_destroy(b)
+
+
+def test_prefetch_hand_worked():
+    """One step ahead: the next batch's evicted blocks come back with victims
+    outside both the next batch and the batch still decoding; the next
+    batch is stamped as used; a prefetch that cannot find room changes
+    nothing; after a prefetch the step itself fetches nothing."""
+    o = ResidencyOracle(8, BT, seed=12, token_bytes=TB)
+    for sid in range(4):
+        o.create(sid, 1000)
+        o.append(sid, 32)      # A, B, C, D: two full blocks each, times 1..4; pool full
+    o.pause(2)                 # C idles
+    o.batch([1, 3])            # B and D decode: time 5
+    a_row, c_row = o.row(0), o.row(2)
+    o.append(1, 16)            # B grows: the LRU block is A's block 0 (time 1)
+    assert o.row(0) == [-1, a_row[1]]
+    assert o.stats["bytes_packed"] == 16 * TB
+    b_new = o.row(1)[2]
+    assert b_new == a_row[0]
+    o.prefetch([0], busy=[1])  # A is next; B still decodes: victim from C (time 3) or D (5)
+    assert o.row(2) == [-1, c_row[1]]                  # C's block 0, the least recent
+    assert o.row(0) == [c_row[0], a_row[1]]
+    assert o.stats["blocks_prefetched"] == 1 and o.stats["prefetches"] == 1
+    assert o.stats["bytes_packed"] == 32 * TB          # + C's 16 tokens, written once
+    assert o.stats["bytes_unpacked"] == 16 * TB        # A's block back
+    assert o.s[0].time > o.s[1].time                   # A stamped after B's append
+    o.batch_reserve([0])       # A's tail is full: one new block (victim C's block 1)
+    assert o.stats["batch_blocks_fetched"] == 0
+    assert o.row(2) == [-1, -1]
+    o.append(3, 16)            # D grows: the LRU outside D is B (its append came before A's stamps)
+    assert o.row(1)[0] == -1
+    before = ([o.row(s) for s in range(4)], list(o.fl.contents()), dict(o.stats))
+    with pytest.raises(NoHotBlocks):
+        o.prefetch([1], busy=[0, 3])       # C holds no hot block: no victim outside A, B, D
+    assert before == ([o.row(s) for s in range(4)], list(o.fl.contents()), dict(o.stats))
+    o.resume(2)
+    o.prefetch([2], busy=[0])  # nothing missing: only the stamp
+    assert o.stats["blocks_prefetched"] == 1 and o.stats["prefetches"] == 2
+
+
+def test_prefetch_then_step_fetches_nothing_without_interference():
+    """Prefetching step k+1's batch during step k leaves step k+1 nothing to
+    fetch when no other allocation comes in between; the blocks it reads
+    are those the prefetch placed."""
+    o = ResidencyOracle(24, BT, seed=14, token_bytes=TB)
+    rnd = random.Random(8)
+    n = 8
+    for sid in range(n):
+        o.create(sid, 10_000)
+        o.append(sid, 32)      # 8 x 2 blocks: 16 of 24
+    cur = [0, 1, 2]
+    done = 0
+    for step in range(80):
+        o.batch_reserve(cur)
+        nxt = sorted(rnd.sample(range(n), k=3))
+        for sid in nxt:        # a paused member of the next batch resumes first
+            if o.s[sid].state == "paused":
+                o.resume(sid)
+        for sid in range(n):   # sessions outside both batches idle
+            if sid not in cur and sid not in nxt and o.s[sid].state == "active":
+                o.pause(sid)
+        try:
+            o.prefetch(nxt, busy=cur)
+        except NoHotBlocks:
+            cur = nxt
+            continue
+        fetched = o.stats["batch_blocks_fetched"]
+        rows = {s: o.row(s) for s in nxt}
+        assert all(x >= 0 for s in nxt for x in rows[s])
+        o.batch_reserve(nxt)
+        assert o.stats["batch_blocks_fetched"] == fetched
+        assert all(o.row(s)[:len(rows[s])] == rows[s] for s in nxt)
+        done += 1
+        cur = nxt
+    assert done > 40
+    assert o.stats["blocks_evicted"] > 0 and o.stats["blocks_prefetched"] > 0

@@ -157,3 +157,66 @@ def test_no_token_written_to_the_cold_tier_twice(tr, mode):
         s = r["stats"]
         assert s["resume_blocks_hit"] + s["resume_blocks_missed"] > 0
         assert s["blocks_evicted"] > 0                # the pool was under pressure
+
+
+def test_lru_trace_with_prefetch_matches_the_residency_oracle(tr, monkeypatch):
+    """The residency-mode schedule with the one-step-ahead prefetch, each pool
+    call mirrored on the residency oracle: block tables, free list and
+    counters equal after every step; the prefetch takes fetches out of the
+    steps themselves without changing the schedule."""
+    import oracle
+    from oracle.residency import NoHotBlocks, ResidencyOracle
+    kv, trace = tr
+    base = small_cfg(trace, lru=True, steps=300)
+    tl = trace.generate(base)
+    peak = trace.plan(dataclasses.replace(base, lru=False), tl)["peak_blocks"]
+    nb = int(math.ceil(1.05 * peak))
+    tok_bytes = base.layers * 2 * base.num_kv_heads * 128 * 2
+    pool, _ = host_pool(kv, base, tl, lru_blocks=nb)
+    o = ResidencyOracle(nb, base.block_tokens, seed=0, token_bytes=tok_bytes)
+    for i, t in enumerate(tl):
+        o.create_paused(i, 1 << 16, t.t0)
+
+    def mirror(name, fn):
+        real = getattr(kv, name)
+
+        def call(*a, **k):
+            err = None
+            try:
+                fn(*a, **k)
+            except NoHotBlocks:
+                err = kv.KV_ERR_NO_HOT_BLOCKS
+            try:
+                real(*a, **k)
+            except kv.KVError as e:
+                assert e.code == err
+                raise
+            assert err is None
+        monkeypatch.setattr(kv, name, call)
+
+    mirror("session_resume", lambda p, sid, st=None: o.resume(sid))
+    mirror("session_pause", lambda p, sid, st=None: o.pause(sid))
+    mirror("session_append", lambda p, sid, k, v, n, st=None: o.append(sid, n))
+    mirror("kv_pool_batch_reserve", lambda p, sids, *a: o.batch_reserve(list(sids)))
+    mirror("kv_pool_prefetch", lambda p, sids, busy=(), st=None: o.prefetch(list(sids), list(busy)))
+    d = trace.TraceDriver(base, pool, tl, gpu=False)
+    try:
+        for k in range(base.steps):
+            d.step(k)
+            assert kv.kv_pool_free_list(pool) == list(o.fl.contents())
+            for i in range(base.sessions):
+                assert kv.session_block_table(pool, i) == o.row(i)
+        st = kv.kv_pool_get_stats(pool)
+        for key, v in o.stats.items():
+            assert st[key] == v, key
+    finally:
+        kv.kv_pool_destroy(pool)
+    assert st["prefetches"] > 0 and st["blocks_evicted"] > 0
+    monkeypatch.undo()
+    # the same schedule without the prefetch: the steps fetch more themselves
+    off = trace.plan(dataclasses.replace(base, prefetch=False), tl, hot_blocks=nb)
+    on = trace.plan(base, tl, hot_blocks=nb)
+    assert on["counts"]["resumes"] == off["counts"]["resumes"]
+    assert on["counts"]["decode_tokens"] == off["counts"]["decode_tokens"]
+    assert on["stats"]["batch_blocks_fetched"] < off["stats"]["batch_blocks_fetched"]
+    assert off["stats"]["blocks_prefetched"] == 0
