@@ -61,6 +61,8 @@ struct Session {
     bool ready_recorded = false;
     cudaEvent_t appended = nullptr;
     bool appended_recorded = false;
+    cudaEvent_t packed = nullptr;     // residency mode: after the last eviction that wrote
+    bool packed_recorded = false;     // the image (it covers every earlier one)
     int16_t pack_fence = -1;          // simple mode: fence slot and generation of the
     uint64_t pack_gen = 0;            // last pause's pack (it reads the table row)
 };
@@ -267,10 +269,16 @@ struct kv_pool {
     }
 
     // Device side of the victims: wait for their last writes, then write the
-    // tokens each image lacks.
+    // tokens each image lacks. A session whose image this writes records its
+    // `packed` event after the writes; the stream first waits for the previous
+    // recording, so the event covers every eviction of the session so far.
+    // Whatever later fetches the session's blocks back waits on it
+    // (wait_packed), on whichever stream it runs.
     int evict_device(const std::vector<Victim> &v, cudaStream_t st) {
-        std::vector<int32_t> seen;
+        std::vector<int32_t> seen, writes;
         for (const Victim &x : v) {
+            if (x.t1 > x.t0 && std::find(writes.begin(), writes.end(), x.sid) == writes.end())
+                writes.push_back(x.sid);
             if (std::find(seen.begin(), seen.end(), x.sid) != seen.end()) continue;
             seen.push_back(x.sid);
             Session &s = sessions[x.sid];
@@ -279,12 +287,31 @@ struct kv_pool {
                 rc = cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s.appended, 0); });
             if (!rc && s.ready_recorded)
                 rc = cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s.ready, 0); });
+            if (!rc) rc = wait_packed(x.sid, st);
             if (rc) return rc;
         }
         std::vector<kvt::BlockJob> jobs;
         for (const Victim &x : v)
             if (x.t1 > x.t0) jobs.push_back(job_for(x.sid, x.j, x.slot, x.t0, x.t1));
-        return run_jobs(jobs, true, st);
+        int rc = run_jobs(jobs, true, st);
+        for (size_t i = 0; !rc && !host_only && i < writes.size(); ++i) {
+            Session &s = sessions[writes[i]];
+            if (!s.packed)
+                rc = cuda("cudaEventCreate",
+                          [&] { return cudaEventCreateWithFlags(&s.packed, cudaEventDisableTiming); });
+            if (!rc) rc = cuda("cudaEventRecord", [&] { return cudaEventRecord(s.packed, st); });
+        }
+        if (rc) return rc;
+        for (int32_t sid : writes) sessions[sid].packed_recorded = !host_only;
+        return KV_OK;
+    }
+
+    // Before blocks of `sid` are fetched from its image on `st`: the image
+    // writes of its evictions (possibly on another stream) must be complete.
+    int wait_packed(int32_t sid, cudaStream_t st) {
+        const Session &s = sessions[sid];
+        if (!s.packed_recorded) return KV_OK;
+        return cuda("cudaStreamWaitEvent", [&] { return cudaStreamWaitEvent(st, s.packed, 0); });
     }
 
     void evict_commit(const std::vector<Victim> &v) {
@@ -465,6 +492,7 @@ int kv_pool_destroy(kv_pool *p) {
         for (auto &s : p->sessions) {
             if (s.ready) cudaEventDestroy(s.ready);
             if (s.appended) cudaEventDestroy(s.appended);
+            if (s.packed) cudaEventDestroy(s.packed);
         }
         for (auto &f : p->fences)
             if (f.ev) cudaEventDestroy(f.ev);
@@ -537,10 +565,11 @@ int session_destroy(kv_pool *p, int32_t sid) {
     p->stats.used_blocks -= freed;
     p->cold_release(s->img_off, s->img_bytes);
     p->stats.cold_bytes_used = p->cold_used;
-    cudaEvent_t ready = s->ready, appended = s->appended;
+    cudaEvent_t ready = s->ready, appended = s->appended, packed = s->packed;
     *s = Session{};
     s->ready = ready;   // events are kept for reuse by the next session in this slot
     s->appended = appended;
+    s->packed = packed;
     return KV_OK;
 }
 
@@ -590,6 +619,7 @@ static int lru_append(kv_pool *p, int32_t sid, const void *k, const void *v, int
     int rc = ensure_event(p, &s->appended);
     if (!rc && s->ready_recorded) rc = wait_event(p, st, s->ready);
     if (!rc) rc = p->evict_device(vic, st);
+    if (!rc && refetch) rc = p->wait_packed(sid, st);
     if (!rc && refetch) {
         rc = p->run_jobs({p->fetch_job(sid, static_cast<int32_t>(tail), got[0], 0,
                                        p->tokens_in_block(*s, tail))}, false, st);
@@ -660,6 +690,7 @@ static int lru_resume(kv_pool *p, int32_t sid, cudaStream_t st) {
     DeviceGuard dg(p->cfg.device, !p->host_only);
     int rc = ensure_event(p, &s->ready);
     if (!rc) rc = p->evict_device(vic, st);
+    if (!rc && need > 0) rc = p->wait_packed(sid, st);
     if (!rc) rc = p->run_jobs(jobs, false, st);
     if (!rc) rc = p->cuda("cudaEventRecord", [&] { return cudaEventRecord(s->ready, st); });
     if (rc) return rc;
@@ -720,6 +751,8 @@ static int lru_fetch(kv_pool *p, const std::vector<int32_t> &uniq,
     for (size_t u = 0; !rc && record_ready && u < uniq.size(); ++u)
         if (!miss[u].empty()) rc = ensure_event(p, &p->sessions[uniq[u]].ready);
     if (!rc) rc = p->evict_device(vic, st);
+    for (size_t u = 0; !rc && u < uniq.size(); ++u)
+        if (!miss[u].empty()) rc = p->wait_packed(uniq[u], st);
     if (!rc) rc = p->run_jobs(jobs, false, st);   // the fetches also write their table entries
     for (size_t u = 0; !rc && record_ready && !p->host_only && u < uniq.size(); ++u)
         if (!miss[u].empty()) {
@@ -1183,6 +1216,8 @@ int kv_pool_batch_reserve(kv_pool *p, const int32_t *sids, int32_t B, int32_t *b
     }
     if (!rc && !fresh.empty()) rc = p->wait_fences(fresh.data(), fresh.size(), st);
     if (!rc) rc = p->evict_device(vic, st);
+    for (int32_t i = 0; !rc && i < B; ++i)
+        if (!miss[i].empty()) rc = p->wait_packed(sids[i], st);
     if (!rc) rc = p->run_jobs(jobs, false, st);
     // Fetched entries were written by their jobs; a new tail block's entry is
     // written by the gather launch below (host-logic pools launch nothing).

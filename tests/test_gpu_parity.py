@@ -453,3 +453,100 @@ def test_config1_scenario(pkg):
     out2 = step()
     assert torch.equal(out1, out2)
     assert pool.check_device() == 0
+
+
+@pytest.mark.parametrize("mig_ctas", [1, 8, 152])
+def test_migration_cta_cap_bit_exact(pkg, mig_ctas):
+    """kv_pool_set_migration_limit caps the migration grids (the copies then
+    walk their items grid-stride with fewer warps): resume-unpack through the
+    one-launch path and the table-reading path (more than 2 048 blocks),
+    append and pause-pack stay bit-exact against the oracle's copies."""
+    dev = torch.device("cuda:0")
+    L, Hkv, bt, seed = 2, 4, 16, 19
+    lens = [700, 33000]
+    NB = sum(-(-t // bt) for t in lens) + 300
+    pool = pkg.Pool(num_layers=L, num_hot_blocks=NB, cold_bytes=(sum(lens) + 2000) * L * 2 * Hkv * 256
+                    + 4096, max_sessions=4, max_batch=8, max_context=34000, alloc_seed=mig_ctas)
+    pool_h = pool.handle
+    pkg.kvtier.kv_pool_set_migration_limit(pool_h, mig_ctas)
+    ref_fl = oracle.FreeList(NB, mig_ctas)
+    hot_ref = np.zeros((NB, L, 2, Hkv, bt, 128), dtype=np.uint16)
+    sids, rows, imgs = [], [], []
+    for T in lens:
+        s = pool.session_create_paused(T + 100, T)
+        synth.fill_image_torch(pool.image(s), seed, s, L, Hkv, 128, T)
+        sids.append(s)
+    torch.cuda.synchronize()
+    for s, T in zip(sids, lens):
+        imgs.append(np_bits(pool.image(s)))
+        pool.session_resume(s)
+        row = ref_fl.pop(-(-T // bt))
+        assert pool.session_block_table(s) == list(row)
+        oracle.unpack(imgs[-1], T, row, hot_ref)
+        rows.append(row)
+    torch.cuda.synchronize()
+    hot = np_bits(pool.hot_view())
+    for row, T in zip(rows, lens):
+        for j, p in enumerate(row):
+            n = min(bt, T - j * bt)
+            assert np.array_equal(hot[p, :, :, :, :n], hot_ref[p, :, :, :, :n])
+    # 50 more tokens each, then the pause packs exactly them
+    for i, (s, T) in enumerate(zip(sids, lens)):
+        k, v = synth.kv_logical_torch(seed + 1, s, range(L), Hkv, 128, T, T + 50, dev)
+        kk, vv = k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+        pool.session_append(s, kk, vv)
+        need = -(-(T + 50) // bt) - len(rows[i])
+        if need > 0:
+            rows[i] = np.concatenate([rows[i], ref_fl.pop(need)])
+        oracle.append(hot_ref, rows[i], T, np_bits(kk), np_bits(vv))
+        pool.session_pause(s)
+        ref_fl.push(rows[i])
+        exp = imgs[i].copy()
+        oracle.pack(hot_ref, rows[i], T, T + 50, exp)
+        torch.cuda.synchronize()
+        assert np.array_equal(np_bits(pool.image(s))[:, :, :, :T + 50], exp[:, :, :, :T + 50])
+    assert pool.free_list() == list(ref_fl.contents())
+    assert pool.check_device() == 0
+    pool.close()
+
+
+@pytest.mark.parametrize("case", ["scale50", "planted64", "planted1024"])
+def test_decode_extreme_logits(pkg, case):
+    """The online softmax's edge cases: scale 50 spreads the logits over
+    hundreds (a near one-hot softmax); a planted key k = c * q (c = 64 or
+    1 024) in a late split puts one token above all others by about 700 or
+    11 600 for the first head of each group, so every other exponent
+    underflows to zero and the merge across splits must still weigh the
+    splits correctly. Outputs must be finite and within the tolerance of
+    the fp64 oracle."""
+    dev = torch.device("cuda:0")
+    lens = [37, 1500, 5000, 17000]
+    pool, sess, tables, q = direct_case(pkg, lens, L=1, seed=40)
+    hot = host_hot(pool, 40, sess, lens, tables)
+    scale = 50.0 if case == "scale50" else 1 / math.sqrt(128)
+    if case.startswith("planted"):
+        c = 64.0 if case == "planted64" else 1024.0
+        hv = pool.hot_view()
+        qc = q.cpu()
+        for b, T in enumerate(lens):
+            t = (3 * T) // 4                      # past the first split when there are several
+            blk, r = int(tables[b, t // 16]), t % 16
+            for g in range(4):
+                kk = (qc[0, b, g * 8].float() * c).to(torch.bfloat16)   # exact: c is 2^k
+                hot[blk, 0, 0, g, r] = kk.view(torch.int16).numpy().view(np.uint16)
+                hv[blk, 0, 0, g, r] = kk.to(dev)
+    pool._scale = scale
+    ref = oracle.paged_decode(hot, q.cpu().view(torch.int16).numpy().view(np.uint16), tables,
+                              lens, scale, 32)
+    got = gpu_decode(pool, -1, q, tables, lens)
+    assert np.all(np.isfinite(got))
+    assert scaled_err(got, ref) <= TOL
+    if case == "planted1024":   # head 0 of each group attends to its planted token alone
+        for b, T in enumerate(lens):
+            t = (3 * T) // 4
+            blk, r = int(tables[b, t // 16]), t % 16
+            v = hot[blk, 0, 1, :, r].astype(np.uint32) << 16
+            v = v.view(np.float32)
+            for g in range(4):
+                assert np.allclose(got[0, b, g * 8], v[g], rtol=1e-5, atol=1e-6)
+    assert pool.check_device() == 0

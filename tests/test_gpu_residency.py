@@ -26,11 +26,13 @@ def bits(t):
     return t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
 
 
-@pytest.mark.parametrize("fused,bt", [(False, 16), (True, 16), (True, 64)])
-def test_residency_random_sequence(cuda_dev, fused, bt):
+@pytest.mark.parametrize("fused,bt,mig_ctas", [(False, 16, 0), (True, 16, 0), (True, 64, 0),
+                                               (True, 16, 1), (True, 64, 8)])
+def test_residency_random_sequence(cuda_dev, fused, bt, mig_ctas):
     """fused: decode batches take their step token with the decode
     (kv_pool_batch_reserve + decode_append_attention, all layers). bt 64:
-    evictions and fetches move 64-token blocks as four 16-token chunks."""
+    evictions and fetches move 64-token blocks as four 16-token chunks.
+    mig_ctas > 0: the evictions and fetches run capped at that many CTAs."""
     import __graft_entry__
     __graft_entry__.build()
     from paper_2609_25782_gb300 import Pool, kvtier
@@ -41,6 +43,7 @@ def test_residency_random_sequence(cuda_dev, fused, bt):
     pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=10 * cap * pool_token_bytes(L, Hkv),
                 max_sessions=10, max_batch=L * 4, max_context=cap, alloc_seed=seed,
                 lru_residency=True, block_tokens=bt)
+    kvtier.kv_pool_set_migration_limit(pool.handle, mig_ctas)
     o = ResidencyOracle(nb, bt, seed=seed, token_bytes=pool.token_bytes)
     rnd = random.Random(seed)
     st = torch.cuda.Stream()
@@ -95,6 +98,17 @@ def test_residency_random_sequence(cuda_dev, fused, bt):
         elif r < 0.7:
             o.pause(sid)
             pool.session_pause(sid, st)
+        elif r < 0.78:          # the next step's blocks ahead of it (same stream here)
+            act = [x for x in live if o.s[x].state == "active"]
+            nxt = rnd.sample(act, k=min(len(act), rnd.randint(1, 3)))
+            busy = rnd.sample(act, k=min(len(act), rnd.randint(0, 2)))
+            try:
+                o.prefetch(nxt, busy)
+            except NoHotBlocks:
+                with pytest.raises(kvtier.KVError):
+                    pool.prefetch(nxt, busy, st)
+                continue
+            pool.prefetch(nxt, busy, st)
         else:
             batch = [x for x in live if o.s[x].state == "active" and
                      (T[x] < cap if fused else T[x] > 0)]
@@ -142,9 +156,9 @@ def test_residency_random_sequence(cuda_dev, fused, bt):
     assert pool.check_device() == 0
     stats = pool.stats()
     for key in ("bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
-                "resume_blocks_missed"):
+                "resume_blocks_missed", "batch_blocks_fetched", "blocks_prefetched"):
         assert stats[key] == o.stats[key], key
-    assert stats["blocks_evicted"] > 10 and checked > 10
+    assert stats["blocks_evicted"] > 10 and checked > 10 and stats["blocks_prefetched"] > 0
     hv = pool.hot_view()
     for sid in live:
         s = o.s[sid]
@@ -166,3 +180,74 @@ def test_residency_random_sequence(cuda_dev, fused, bt):
 
 def pool_token_bytes(L, Hkv):
     return L * 2 * Hkv * 128 * 2
+
+
+def test_fetch_waits_for_an_eviction_on_another_stream(cuda_dev):
+    """A block evicted on one stream (its tokens written to the image) and
+    fetched back on another must be fetched after that write. Stream A is
+    held back by a spin before a resume that evicts all of session Y's
+    blocks; stream B then batches Y, fetching them from Y's image, and
+    decodes. A fetch that did not wait would read the image before the
+    eviction wrote it."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool
+
+    L, Hq, Hkv, D, bt, seed, cap = 2, 32, 4, 128, 16, 31, 64
+    pool = Pool(num_layers=L, num_hot_blocks=6, cold_bytes=4 * cap * pool_token_bytes(L, Hkv),
+                max_sessions=4, max_batch=L, max_context=cap, alloc_seed=seed,
+                lru_residency=True)
+    o = ResidencyOracle(6, bt, seed=seed, token_bytes=pool.token_bytes)
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def append(sid, n):
+        with torch.cuda.stream(sa):
+            k, v = synth.kv_logical_torch(seed, sid, range(L), Hkv, D, 0, n, cuda_dev)
+            pool.session_append(sid, k.permute(0, 2, 1, 3).contiguous(),
+                                v.permute(0, 2, 1, 3).contiguous(), sa)
+
+    y = pool.session_create(cap)
+    o.create(y, cap)
+    append(y, 40)                       # three blocks, none of them in the image yet
+    o.append(y, 40)
+    x = pool.session_create_paused(cap, 48)
+    o.create_paused(x, cap, 48)
+    with torch.cuda.stream(sa):
+        synth.fill_image_torch(pool.image(x), seed, x, L, Hkv, D, 48)
+    z = pool.session_create(cap)
+    o.create(z, cap)
+    append(z, 48)                       # the pool is full
+    o.append(z, 48)
+    q = synth.queries_torch(seed, [y], range(L), Hq, D, cuda_dev)
+    mb = cap // bt
+    tables = torch.empty(1, mb, dtype=torch.int32, device=cuda_dev)
+    slens = torch.empty(1, dtype=torch.int32, device=cuda_dev)
+    out = torch.full((L, 1, Hq, D), float("nan"), dtype=torch.float32, device=cuda_dev)
+    torch.cuda.synchronize()
+
+    with torch.cuda.stream(sa):
+        torch.cuda._sleep(200_000_000)  # about 0.1 s of stream A before the eviction
+    pool.session_resume(x, sa)          # evicts Y's three blocks, writing its 40 tokens
+    o.resume(x)
+    assert o.row(y) == [-1, -1, -1] and o.stats["bytes_packed"] == 40 * pool.token_bytes
+    pool.batch_tables([y], tables, mb, slens, sb)    # Y's blocks back from its image
+    o.batch([y])
+    pool.decode_attention(-1, q, tables, slens, 1, mb, 1 / math.sqrt(D), out, sb)
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    assert pool.session_block_table(y) == o.row(y)
+    rows = np.full((1, mb), -1, dtype=np.int32)
+    rows[0, :3] = o.row(y)
+    hot = synth.hot_pool_np(seed, [y], [40], rows, 6, L, Hkv, D, bt)
+    ref = oracle.paged_decode(hot, bits(q), rows, [40], 1 / math.sqrt(D), Hq)
+    got = out.double().cpu().numpy()
+    assert np.all(np.isfinite(got))
+    assert np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref))) <= TOL
+    k, v = synth.session_kv_np(seed, y, range(L), Hkv, D, 40)
+    hv = pool.hot_view()
+    for j, slot in enumerate(o.row(y)):
+        n = min(bt, 40 - j * bt)
+        hb = bits(hv[slot])
+        assert np.array_equal(hb[:, 0, :, :n], k[:, :, j * bt:j * bt + n])
+        assert np.array_equal(hb[:, 1, :, :n], v[:, :, j * bt:j * bt + n])
+    pool.close()

@@ -20,7 +20,10 @@ pytestmark = pytest.mark.gpu
 TOL = 1e-2
 
 
-def test_small_trace_parity(cuda_dev):
+@pytest.mark.parametrize("lead", [1, 2])
+def test_small_trace_parity(cuda_dev, lead):
+    """lead: steps between a session's resume and its first decode (2: the
+    admitted session waits a step longer, its resume further ahead)."""
     import __graft_entry__
     __graft_entry__.build()
     from paper_2609_25782_gb300 import Pool, kvtier
@@ -28,7 +31,7 @@ def test_small_trace_parity(cuda_dev):
 
     cfg = tr.TraceConfig(sessions=6, t0_min=100, t0_max=700, burst_mean=8.0, pause_mean_s=0.6,
                          append_median=40.0, append_sigma=1.0, append_max=300, active_cap=2,
-                         steps=150, dt_s=0.1, layers=2, seed=5)
+                         steps=150, dt_s=0.1, layers=2, seed=5, admit_lead=lead)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     assert plan["counts"]["pauses"] >= 10
@@ -169,13 +172,17 @@ def test_full_trace_sampled_parity(cuda_dev):
     pool.close()
 
 
-def test_small_trace_residency_under_pressure(cuda_dev):
+@pytest.mark.parametrize("prefetch,lead", [(True, 1), (False, 1), (True, 2)])
+def test_small_trace_residency_under_pressure(cuda_dev, prefetch, lead):
     """The small trace in residency mode (LRU, write-on-evict) with a hot pool
     of exactly the simple mode's peak: paused sessions' blocks are evicted and
     fetched back, step tokens go through the fused decode. At sampled steps
     the decode must match the oracle over the members' logical KV (so every
     block fetched back holds the right bytes), and the run's counters must
-    equal the residency dry run's."""
+    equal the residency dry run's. Without the one-step-ahead prefetch some
+    blocks are fetched inside the steps (victims of admissions on the
+    migration stream), which exercises fetches after evictions made on the
+    other stream."""
     import dataclasses
 
     import __graft_entry__
@@ -185,13 +192,16 @@ def test_small_trace_residency_under_pressure(cuda_dev):
 
     base = tr.TraceConfig(sessions=6, t0_min=100, t0_max=700, burst_mean=8.0, pause_mean_s=0.6,
                           append_median=40.0, append_sigma=1.0, append_max=300, active_cap=2,
-                          steps=150, dt_s=0.1, layers=2, seed=5)
+                          steps=150, dt_s=0.1, layers=2, seed=5, admit_lead=lead)
     trace = tr.generate(base)
     simple = tr.plan(base, trace)
-    cfg = dataclasses.replace(base, lru=True)
+    cfg = dataclasses.replace(base, lru=True, prefetch=prefetch)
     nb = simple["peak_blocks"]
     dry = tr.plan(cfg, trace, hot_blocks=nb)["stats"]
     assert dry["blocks_evicted"] > 0 and dry["resume_blocks_missed"] > 0
+    assert (dry["prefetches"] > 0) == prefetch
+    if not prefetch:
+        assert dry["batch_blocks_fetched"] > 0
     L, Hkv, Hq, D, bt = cfg.layers, cfg.num_kv_heads, cfg.num_q_heads, 128, cfg.block_tokens
     pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=simple["cold_bytes"] + 4096,
                 max_sessions=cfg.sessions, max_batch=cfg.active_cap,
@@ -239,6 +249,7 @@ def test_small_trace_residency_under_pressure(cuda_dev):
     assert pool.check_device() == 0
     st = pool.stats()
     for key in ("bytes_packed", "bytes_unpacked", "blocks_evicted", "resume_blocks_hit",
-                "resume_blocks_missed", "resumes", "pauses"):
+                "resume_blocks_missed", "resumes", "pauses", "batch_blocks_fetched",
+                "blocks_prefetched", "prefetches"):
         assert st[key] == dry[key], key
     pool.close()
