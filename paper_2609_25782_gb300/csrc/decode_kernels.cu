@@ -685,17 +685,21 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
 }  // namespace
 
 bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why) {
-    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-    if (!encode) {
+    // Resolved once; a function-local static is initialised exactly once even
+    // when pools are created, or allocation-free decodes issued, on several
+    // host threads at the same moment.
+    static const PFN_cuTensorMapEncodeTiled_v12000 encode = [] {
         void *fn = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
                                              cudaEnableDefault, &q) != cudaSuccess ||
-            q != cudaDriverEntryPointSuccess || !fn) {
-            *why = "cuTensorMapEncodeTiled entry point unavailable";
-            return false;
-        }
-        encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+            q != cudaDriverEntryPointSuccess)
+            fn = nullptr;
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }();
+    if (!encode) {
+        *why = "cuTensorMapEncodeTiled entry point unavailable";
+        return false;
     }
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(kRowBytes)};

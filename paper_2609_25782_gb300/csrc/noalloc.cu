@@ -20,10 +20,22 @@ constexpr int kMaxDevices = 64;
 // Partials (fp32 accumulators, then (max, sum) pairs), then one flag word.
 static __device__ __align__(256) unsigned char g_decode_scratch[KV_NOALLOC_SCRATCH_BYTES];
 
+// Tensor maps of the hot arenas a device's calls have used, so that a call
+// over an arena seen before skips the encode (a driver call per decode).
+constexpr int kMapCache = 4;
+struct CachedMap {
+    const void *base = nullptr;
+    int64_t rows = 0;
+    uint64_t last_use = 0;
+    CUtensorMap map{};
+};
+
 struct DeviceScratch {
     unsigned char *ptr = nullptr;   // device address of g_decode_scratch
     int num_sms = 1;
     bool ready = false;
+    CachedMap maps[kMapCache];
+    uint64_t clock = 0;
 };
 DeviceScratch g_dev[kMaxDevices];
 std::mutex g_mu;
@@ -52,6 +64,31 @@ int setup_device(int dev, unsigned char **ptr, int *num_sms) {
     }
     *ptr = d.ptr;
     *num_sms = d.num_sms;
+    return KV_OK;
+}
+
+// The hot arena's tensor map for this device: from the cache, else encoded
+// and put in place of the least recently used entry.
+int device_tensor_map(int dev, void *hot_base, int64_t rows, CUtensorMap *out) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    DeviceScratch &d = g_dev[dev];
+    CachedMap *victim = &d.maps[0];
+    for (CachedMap &m : d.maps) {
+        if (m.base == hot_base && m.rows == rows) {
+            m.last_use = ++d.clock;
+            *out = m.map;
+            return KV_OK;
+        }
+        if (m.last_use < victim->last_use) victim = &m;
+    }
+    const char *why = nullptr;
+    CUtensorMap map;
+    if (!kvt::encode_hot_tensor_map(&map, hot_base, rows, &why)) return fail(KV_ERR_CUDA, why);
+    victim->base = hot_base;
+    victim->rows = rows;
+    victim->map = map;
+    victim->last_use = ++d.clock;
+    *out = map;
     return KV_OK;
 }
 
@@ -115,15 +152,15 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     int rc = setup_device(c.device, &scratch, &num_sms);
     if (rc) return rc;
     CUtensorMap map;
-    const char *why = nullptr;
-    if (!kvt::encode_hot_tensor_map(&map, c.hot_base, rows, &why)) return fail(KV_ERR_CUDA, why);
+    rc = device_tensor_map(c.device, c.hot_base, rows, &map);
+    if (rc) return rc;
 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // The kernels OR their bounds-check bits into this word. Nothing reads it
+    // (this entry point has no pool to report through), so it needs no
+    // clearing; no scratch has to start at zero, since every partial is
+    // written before it is read within the call.
     int32_t *flag = reinterpret_cast<int32_t *>(scratch + KV_NOALLOC_SCRATCH_BYTES - 256);
-    // The flag word is the only scratch that must start at zero; partials are
-    // written before they are read within the call.
-    if (cudaMemsetAsync(flag, 0, sizeof(int32_t), st) != cudaSuccess)
-        return fail(KV_ERR_CUDA, "decode_attention_noalloc: cudaMemsetAsync failed");
 
     kvt::DecodeArgs a;
     a.q = static_cast<const uint16_t *>(q);
