@@ -453,7 +453,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     cfg = tr.TraceConfig(seed=replica_seed(args.seed, rank), steps=args.trace_steps,
                          admit_lead=args.trace_admit_lead,
                          fused_append=not args.trace_unfused_append,
-                         prefetch=not args.trace_no_prefetch)
+                         prefetch=not args.trace_no_prefetch,
+                         overlap=not args.trace_no_overlap, max_ahead=args.trace_max_ahead)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -632,25 +633,35 @@ def run_trace(args, rank, lru_factor: float = 0.0):
 SWEEP_B = (1, 8, 32, 128, 256)
 SWEEP_T = (1024, 4096, 16384, 65536, 131072)
 SWEEP_CAP = 120e9
+# The bounded curve every default run reports (a subset of the full sweep):
+# (block tokens, batch, context) decode points and resume-unpack contexts.
+CURVE_DECODE = ((16, 1, 16384), (16, 1, 131072), (16, 8, 4096), (16, 8, 65536),
+                (16, 32, 16384), (16, 256, 4096), (64, 1, 16384), (64, 8, 65536))
+CURVE_RESUME = (1024, 131072)
 
 
-def run_sweep(args):
-    """Roofline-fraction curve: the resume-unpack sweep over single sessions of
-    1K..128K tokens, then decode over (block size, batch, context) with total
-    KV <= 120 GB, per-layer launches and the all-layers launch."""
+def run_sweep(args, decode_points=None, resume_T=SWEEP_T):
+    """Roofline-fraction curve: the resume-unpack sweep over single sessions
+    (1K..128K tokens by default), then decode over (block size, batch,
+    context) with total KV <= 120 GB, per-layer launches and the all-layers
+    launch. decode_points: (bt, B, T) triples, default every point of the
+    full grid."""
     import torch
     import synth
     from paper_2609_25782_gb300 import Pool, kvtier
     dev = torch.device("cuda", torch.cuda.current_device())
     peak, _ = hbm_peak()
+    if decode_points is None:
+        decode_points = [(bt, B, T) for bt in (16, 64) for B in SWEEP_B for T in SWEEP_T
+                         if B * T * TOKEN_BYTES <= SWEEP_CAP]
     # resume-unpack sweep (first, before the long decode sweep loads the GPU)
     resume = []
-    Tm = max(SWEEP_T)
+    Tm = max(resume_T)
     pool = Pool(num_layers=L, num_hot_blocks=Tm // 16 + 64, cold_bytes=Tm * TOKEN_BYTES * 2 + 4096,
-                max_sessions=len(SWEEP_T) + 1, max_batch=4, max_context=Tm, alloc_seed=args.seed,
+                max_sessions=len(resume_T) + 1, max_batch=4, max_context=Tm, alloc_seed=args.seed,
                 device=dev.index)
     stream = torch.cuda.Stream(device=dev)
-    for T in SWEEP_T:
+    for T in resume_T:
         s = pool.session_create_paused(T, T)
         synth.fill_image_torch(pool.image(s), args.seed, s, L, HKV, D, T)
         ms, ms_idle = [], []
@@ -679,15 +690,15 @@ def run_sweep(args):
     torch.cuda.empty_cache()
     scale = 1 / math.sqrt(D)
     points = []
-    for bt in (16, 64):
-        pts = [(B, T) for B in SWEEP_B for T in SWEEP_T if B * T * TOKEN_BYTES <= SWEEP_CAP]
+    for bt in sorted({p[0] for p in decode_points}):
+        pts = [(B, T) for b2, B, T in decode_points if b2 == bt]
         max_tok = max(B * T for B, T in pts)
         nb = max_tok // bt + 64
         Bmax = max(B for B, _ in pts)
         # workspace rows: the largest of layers x B x Hq x S(T) over the points
         splits = kvtier.kv_decode_splits
         need = max(L * B * HQ * splits(T) for B, T in pts)
-        ctx = max(SWEEP_T)
+        ctx = max(T for _, T in pts)
         pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=256, block_tokens=bt,
                     max_sessions=4, max_batch=-(-need // (HQ * splits(ctx))),
                     max_context=ctx, device=dev.index)
@@ -881,6 +892,10 @@ def main():
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--only-trace", action="store_true",
                     help="run only the agentic trace (simple and residency modes)")
+    ap.add_argument("--trace-max-ahead", type=int, default=3,
+                    help="trace: steps the host may run ahead of the GPU (0: unbounded)")
+    ap.add_argument("--trace-no-overlap", action="store_true",
+                    help="trace: launch every layer's decode fully serialised")
     ap.add_argument("--trace-no-prefetch", action="store_true",
                     help="trace (residency mode): no one-step-ahead fetch of spilled blocks")
     ap.add_argument("--trace-lru-factor", type=float, default=1.5,
@@ -888,6 +903,8 @@ def main():
     ap.add_argument("--trace-unfused-append", action="store_true",
                     help="trace: write each step's token with its own kernel before the decode")
     ap.add_argument("--no-trace", action="store_true")
+    ap.add_argument("--no-curve", action="store_true",
+                    help="skip the bounded roofline curve in the secondary results")
     ap.add_argument("--graph", action=argparse.BooleanOptionalAction, default=True,
                     help="replay the per-layer calls of a step from one CUDA graph")
     ap.add_argument("--no-overlap", action="store_true",
@@ -960,6 +977,11 @@ def main():
     if secondary is not None and not args.no_trace:
         secondary["trace"] = run_trace(args, rank)
         secondary["trace_lru"] = run_trace(args, rank, lru_factor=args.trace_lru_factor)
+    if secondary is not None and not args.no_curve:
+        # the bounded roofline curve (config 5 subset); --sweep prints the full grid
+        t_curve = time.time()
+        secondary["sweep"] = run_sweep(args, decode_points=CURVE_DECODE, resume_T=CURVE_RESUME)
+        secondary["sweep"]["seconds"] = round(time.time() - t_curve, 1)
     nl, nbatch = args.layers, args.batch
     headline = (nl, nbatch, args.tmin, args.tmax) == (L, B2, TMIN2, TMAX2)
 

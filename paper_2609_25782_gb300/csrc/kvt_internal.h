@@ -32,9 +32,12 @@ constexpr int32_t kErrTimeout = 4;     // an mbarrier wait gave up
 #ifndef KVT_SPLIT_MAX_TILES
 #define KVT_SPLIT_MAX_TILES 128
 #endif
+#ifndef KVT_SPLIT_TARGET
+#define KVT_SPLIT_TARGET 16       // splits per (session, kv-head) while the clamp is inactive
+#endif
 __host__ __device__ inline int tiles_of(int T) { return (T + kTileTokens - 1) / kTileTokens; }
 __host__ __device__ inline int split_tiles(int T) {
-    int s = (tiles_of(T) + 15) / 16;   // aim at 16 splits per (session, kv-head)
+    int s = (tiles_of(T) + KVT_SPLIT_TARGET - 1) / KVT_SPLIT_TARGET;
     return s < KVT_SPLIT_MIN_TILES ? KVT_SPLIT_MIN_TILES
                                    : (s > KVT_SPLIT_MAX_TILES ? KVT_SPLIT_MAX_TILES : s);
 }
@@ -42,14 +45,15 @@ __host__ __device__ inline int num_splits(int T) {
     int st = split_tiles(T);
     return (tiles_of(T) + st - 1) / st;
 }
-// Upper bound of num_splits(T) for T <= max_tokens. Below 16*min tiles the
-// split is min tiles (ceil(tiles/min) splits, fewer than 16); while the clamp
-// is inactive there are at most 16; above 16*max tiles, ceil(tiles/max).
+// Upper bound of num_splits(T) for T <= max_tokens. Below target*min tiles
+// the split is min tiles (ceil(tiles/min) splits, fewer than the target);
+// while the clamp is inactive there are at most `target`; above target*max
+// tiles, ceil(tiles/max).
 inline int max_splits_for(int64_t max_tokens) {
     const int64_t tiles = (max_tokens + kTileTokens - 1) / kTileTokens;
     const int64_t at_max = (tiles + KVT_SPLIT_MAX_TILES - 1) / KVT_SPLIT_MAX_TILES;
     int64_t at_min = (tiles + KVT_SPLIT_MIN_TILES - 1) / KVT_SPLIT_MIN_TILES;
-    if (at_min > 16) at_min = 16;
+    if (at_min > KVT_SPLIT_TARGET) at_min = KVT_SPLIT_TARGET;
     return (int)(at_max > at_min ? at_max : at_min);
 }
 

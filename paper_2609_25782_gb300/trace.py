@@ -54,6 +54,12 @@ class TraceConfig:
     admit_lead: int = 1              # steps between a resume and the session's first decode
     fused_append: bool = True        # step token written by the decode kernel itself
     prefetch: bool = True            # residency mode: next step's spilled blocks fetched ahead
+    overlap: bool = True             # layer l > 0 starts while layer l-1's call drains
+    # The host issues step k only after step k - max_ahead has finished on the
+    # GPU (as a serving loop that reads back a step's tokens would); 0: never
+    # waits. A host that runs further ahead fills the CUDA launch queue, and a
+    # launch that waits for queue space can stall the host for tens of ms.
+    max_ahead: int = 3
 
 
 @dataclass
@@ -173,6 +179,8 @@ class TraceDriver:
     # ------------------------------------------------------------------- step
     def step(self, k: int) -> None:
         cfg = self.cfg
+        if self.gpu and cfg.max_ahead > 0 and len(self.step_events) >= cfg.max_ahead:
+            self.step_events[-cfg.max_ahead][1].synchronize()
         h0 = time.perf_counter()
         h_adm = h_res = None
         now = k * cfg.dt_s
@@ -263,7 +271,7 @@ class TraceDriver:
                 for l in range(cfg.layers):
                     # layer l > 0 follows layer l-1's call, which writes only `out`
                     # and (fused) layer l-1's rows of the pool
-                    flags = kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 else 0
+                    flags = kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 and cfg.overlap else 0
                     if cfg.fused_append:
                         kvtier.decode_append_attention(
                             self.pool, l, self.q[l], k_new[l], v_new[l], self.tables,
