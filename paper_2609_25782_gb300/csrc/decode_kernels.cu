@@ -21,31 +21,37 @@
 namespace kvt {
 namespace {
 
-#ifndef KVT_DECODE_WARPS
-#define KVT_DECODE_WARPS 4
-#endif
 #ifndef KVT_STAGES
 #define KVT_STAGES 2   // 4 warps x 2 x 8 KiB: 3 CTAs (24 tiles in flight) per SM
 #endif
-constexpr int kDecodeWarps = KVT_DECODE_WARPS;
 constexpr int kCombineWarps = 4;
 constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
 constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
-// Ring depths (tiles in flight per warp) by how many CTAs share an SM: a
-// grid that fills every SM three times over runs 3 CTAs of KVT_STAGES slots
-// per SM; smaller grids get deeper rings so each SM still keeps ~24 tiles
-// in flight. The depth changes only the prefetch distance, never which warp
-// takes which tile, so all variants give bit-identical results.
+// The plan of one split: its tiles are dealt round robin to kAccs running
+// softmax states (accumulator v takes tiles v, v + kAccs, ...), which merge
+// in the order v = 0 .. kAccs-1 at the end. That plan fixes the result; how
+// the accumulators map to warps is a launch choice:
+//   <4 warps, KVT_STAGES slots>  3 CTAs per SM; a warp owns accumulators w
+//                                and w + 4 and alternates between them, so
+//                                consecutive tiles of a warp are independent
+//   <4 warps, 3 slots>           2 CTAs per SM
+//   <8 warps, 3 slots>           1 CTA per SM (small grids): one accumulator
+//                                per warp, twice the warps per SM
+// Each SM keeps about 24 tiles in flight whatever the variant, and every
+// variant gives bit-identical results.
+constexpr int kAccs = 8;
 #ifndef KVT_WAVE_MARGIN
 #define KVT_WAVE_MARGIN 0.1   // last-wave fill gain that moves a grid to 2 CTAs per SM
 #endif
+constexpr int kWarpsNarrow = 4, kWarpsWide = 8;
 constexpr int kStagesFull = KVT_STAGES;    // 3 CTAs per SM
 constexpr int kStagesHalf = 3;             // 2 CTAs per SM
-constexpr int kStagesOne = 6;              // 1 CTA per SM
-__host__ __device__ constexpr int decode_smem(int stages) {
-    return kDecodeWarps * stages * kTileBytes + 1024 + 256;   // rings, alignment, barriers
+constexpr int kStagesOne = 3;              // 1 CTA per SM (8 warps)
+__host__ __device__ constexpr int decode_smem(int warps, int stages) {
+    return warps * stages * kTileBytes + 1024 + 256;   // rings, alignment, barriers
 }
-static_assert(kDecodeWarps * kStagesOne * 8 <= 256, "mbarriers must fit their 256-byte area");
+static_assert(kWarpsWide * kStagesOne * 8 <= 256, "mbarriers must fit their 256-byte area");
+static_assert(kWarpsNarrow * kStagesHalf * 8 <= 256, "mbarriers must fit their 256-byte area");
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;   // 2 s
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -149,21 +155,31 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 
 // ---------------------------------------------------------------------------
 // K1: one CTA = (split s, kv-head g, layer-batch row lb = li*B + b).
-// Warp w consumes the split's tiles w, w+4, ... through its own ring of
-// kStages 8 KiB slots. Per tile (16 tokens):
+// The split's tiles go round robin to kAccs = 8 accumulators; warp w of the
+// kWarps consumes tiles w, w + kWarps, ... through its own ring of kStages
+// 8 KiB slots, tile k of the warp feeding its accumulator k % (8 / kWarps).
+// Per tile (16 tokens):
 //   S^T[16 tok x 8 heads] = K[16 x 128] . Q^T       8 x mma m16n8k16
 //   online softmax over tokens (columns = heads)
 //   O^T[128 x 8] += V^T[128 x 16] . P^T[16 x 8]     8 x mma, P^T via movmatrix
-// The four warps' states merge in shared memory in warp order; a one-split
+// The accumulators merge in shared memory in accumulator order; a one-split
 // session writes its normalised output, others write (m, l, acc) partials.
 // ---------------------------------------------------------------------------
-template <int kStages>
-__global__ void __launch_bounds__(kDecodeWarps * 32)
+struct AccState {
+    float m0, m1;   // running max, heads 2(lane%4) and +1 (log2 units)
+    float l0, l1;   // this lane's share of the normaliser
+    float o[8][4];  // O^T fragments
+};
+
+template <int kWarps, int kStages>
+__global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages == kStagesFull ? 3 : 1)
     decode_split_kernel(const __grid_constant__ CUtensorMap map, const DecodeArgs a) {
+    constexpr int kA = kAccs / kWarps;   // accumulators per warp
+    static_assert(kA * kWarps == kAccs, "accumulators divide among the warps");
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kDecodeWarps * kStages * kTileBytes);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kWarps * kStages * kTileBytes);
 
     // The grid is (splits, kv-heads, rows); its blocks go out in linear order,
     // read here head-fastest so the CTAs of one split's kv-heads, whose runs
@@ -186,15 +202,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     // started; it still waits for this grid to finish before reading.
     asm volatile("griddepcontrol.launch_dependents;");
     const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
-    // Tables at most 16 x KVT_SPLIT_MIN_TILES tiles wide split every session
-    // every KVT_SPLIT_MIN_TILES tiles, so this warp's tiles are known before
-    // T: their block ids load alongside T instead of after it. Lanes past
-    // the session's tiles may read table entries past its blocks (never used).
-    constexpr int kMinWarpTiles = KVT_SPLIT_MIN_TILES / kDecodeWarps;
+    // Tables at most KVT_SPLIT_TARGET x KVT_SPLIT_MIN_TILES tiles wide split
+    // every session every KVT_SPLIT_MIN_TILES tiles, so this warp's tiles are
+    // known before T: their block ids load alongside T instead of after it.
+    // Lanes past the session's tiles may read table entries past its blocks
+    // (never used).
+    constexpr int kMinWarpTiles = KVT_SPLIT_MIN_TILES / kWarps;
     const bool fixed_split = split_tiles(a.max_blocks * sh.bt) == KVT_SPLIT_MIN_TILES;
     int early_blk = 0;
     if (fixed_split && lane < kMinWarpTiles) {
-        const int j = (split * KVT_SPLIT_MIN_TILES + warp + lane * kDecodeWarps) * kTileTokens / sh.bt;
+        const int j = (split * KVT_SPLIT_MIN_TILES + warp + lane * kWarps) * kTileTokens / sh.bt;
         if (j < a.max_blocks) early_blk = trow[j];
     }
     const int T = a.seq_lens[b];
@@ -207,7 +224,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     const int st = split_tiles(T);
     const int tile0 = split * st;
     const int tile1 = min(tiles_of(T), tile0 + st);
-    const int my_tiles = (tile1 - tile0 - warp + kDecodeWarps - 1) / kDecodeWarps;  // may be <= 0
+    const int my_tiles = (tile1 - tile0 - warp + kWarps - 1) / kWarps;  // may be <= 0
 
     uint8_t *ring = smem + warp * kStages * kTileBytes;
     const uint32_t ring_s = smem_u32(ring);
@@ -217,12 +234,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     // Block ids of this warp's tiles, fetched together up front: lane t
     // holds the block of the warp's tile t, so no table load waits in front
     // of a tile copy (one CTA per SM has no other warps to hide it behind).
-    static_assert((KVT_SPLIT_MAX_TILES + kDecodeWarps - 1) / kDecodeWarps <= 32,
+    static_assert((KVT_SPLIT_MAX_TILES + kWarps - 1) / kWarps <= 32,
                   "a warp's tiles of one split must fit one block id per lane");
-    static_assert(KVT_SPLIT_MIN_TILES % kDecodeWarps == 0, "whole tiles per warp");
+    static_assert(KVT_SPLIT_MIN_TILES % kWarps == 0, "whole tiles per warp");
     int lane_blk = early_blk;
     if (!fixed_split && lane < my_tiles)
-        lane_blk = trow[(tile0 + warp + lane * kDecodeWarps) * kTileTokens / sh.bt];
+        lane_blk = trow[(tile0 + warp + lane * kWarps) * kTileTokens / sh.bt];
 
     if (lane == 0) {
         for (int i = 0; i < kStages; ++i) mbar_init(bar0 + 8 * i, 1);
@@ -233,7 +250,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     // Producer step (lane 0): tile k of this warp, in block blk, into slot
     // k % kStages.
     auto issue = [&](int k, int blk) {
-        const int ti = tile0 + warp + k * kDecodeWarps;
+        const int ti = tile0 + warp + k * kWarps;
         const int tok = ti * kTileTokens;
         const int j = tok / sh.bt;
         if (blk < 0 || blk >= sh.num_blocks) {
@@ -283,11 +300,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         }
     }
 
-    float m0 = -INFINITY, m1 = -INFINITY;   // running max, heads 2(lane%4) and +1
-    float l0 = 0.f, l1 = 0.f;               // this lane's share of the normaliser
-    float o[8][4];
+    AccState acc_state[kA];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+    for (int i = 0; i < kA; ++i) {
+        acc_state[i].m0 = acc_state[i].m1 = -INFINITY;
+        acc_state[i].l0 = acc_state[i].l1 = 0.f;
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            acc_state[i].o[r][0] = acc_state[i].o[r][1] = acc_state[i].o[r][2] = acc_state[i].o[r][3] = 0.f;
+    }
     const float sl = a.scale_log2;
     int fail_k = -1;
 
@@ -338,31 +359,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         x[2] = v1 ? (sa[2] + sb[2]) * sl : -INFINITY;
         x[3] = v1 ? (sa[3] + sb[3]) * sl : -INFINITY;
     };
-    // Online-softmax step of one tile given its column maxima: advances m and
-    // l, returns P (rounded to bf16, as the PV product sees it) and the
-    // factors that rescale the accumulator.
-    auto softmax_step = [&](const float (&x)[4], float mx0, float mx1, uint32_t &p01,
-                            uint32_t &p23, float &al0, float &al1) {
-        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        al0 = ex2(m0 - mn0);
-        al1 = ex2(m1 - mn1);
-        m0 = mn0;
-        m1 = mn1;
-        float q0, q1, q2, q3;
-        p01 = pack_bf16(ex2(x[0] - mn0), ex2(x[1] - mn1), q0, q1);
-        p23 = pack_bf16(ex2(x[2] - mn0), ex2(x[3] - mn1), q2, q3);
-        l0 = l0 * al0 + q0 + q2;
-        l1 = l1 * al1 + q1 + q3;
-    };
-    auto rescale = [&](float al0, float al1) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            o[i][0] *= al0;
-            o[i][1] *= al1;
-            o[i][2] *= al0;
-            o[i][3] *= al1;
-        }
-    };
     // Last, partial tile: slots past T may hold anything (NaN); P is 0 there
     // but 0 * NaN is not, so clear those V rows of tile k.
     auto clear_tail_v = [&](int k, int tok_base) {
@@ -380,12 +376,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             __syncwarp();
         }
     };
-    auto tile_base = [&](int k) { return (tile0 + warp + k * kDecodeWarps) * kTileTokens; };
-    auto slot_of = [&](int k) { return ring_s + (k % kStages) * kTileBytes; };
+    auto tile_base = [&](int k) { return (tile0 + warp + k * kWarps) * kTileTokens; };
 
-    // One tile: scores, softmax, O^T += V^T . P^T. False: its wait timed out.
-    auto one_tile = [&](int k) -> bool {
-        const uint32_t slot = slot_of(k);
+    // One tile into accumulator s: scores, softmax, O^T += V^T . P^T.
+    // False: its wait timed out.
+    auto one_tile = [&](int k, AccState &s) -> bool {
+        const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
         if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) return false;
         const int tok_base = tile_base(k);
         if (a.k_new != nullptr && tok_base + kTileTokens >= T) splice_new(k, tok_base);
@@ -405,10 +401,24 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
             mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
         }
-        uint32_t p01, p23;
-        float al0, al1;
-        softmax_step(x, mx0, mx1, p01, p23, al0, al1);
-        rescale(al0, al1);
+        // Online-softmax step: advance m and l, P rounded to bf16 (as the PV
+        // product sees it), the accumulator rescaled.
+        const float mn0 = fmaxf(s.m0, mx0), mn1 = fmaxf(s.m1, mx1);
+        const float al0 = ex2(s.m0 - mn0), al1 = ex2(s.m1 - mn1);
+        s.m0 = mn0;
+        s.m1 = mn1;
+        float q0, q1, q2, q3;
+        const uint32_t p01 = pack_bf16(ex2(x[0] - mn0), ex2(x[1] - mn1), q0, q1);
+        const uint32_t p23 = pack_bf16(ex2(x[2] - mn0), ex2(x[3] - mn1), q2, q3);
+        s.l0 = s.l0 * al0 + q0 + q2;
+        s.l1 = s.l1 * al1 + q1 + q3;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            s.o[i][0] *= al0;
+            s.o[i][1] *= al1;
+            s.o[i][2] *= al0;
+            s.o[i][3] *= al1;
+        }
         const uint32_t pb0 = movmatrix_t(p01);   // P^T tokens 0-7  -> B fragment
         const uint32_t pb1 = movmatrix_t(p23);   // P^T tokens 8-15
         clear_tail_v(k, tok_base);
@@ -418,7 +428,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             uint32_t r0, r1, r2, r3;
             const int u = 2 * i + vhi;
             ldsm_x4_t(vslot + (u >> 3) * kHalfBytes + swz(vrow, u & 7), r0, r1, r2, r3);
-            mma_bf16(o[i], r0, r1, r2, r3, pb0, pb1);
+            mma_bf16(s.o[i], r0, r1, r2, r3, pb0, pb1);
         }
         __syncwarp();
         const int nblk = blk_of(k + kStages);
@@ -426,86 +436,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         return true;
     };
 
-    // Tiles k and k+1 together (one CTA per SM, where each warp's own
-    // dependent mma/shuffle latency is the limit): the two tiles' score
-    // products and column maxima run as independent chains, and tile k+1's V
-    // fragments are loaded before tile k's product lands. The state updates
-    // (m, l, then O) are applied tile k first, exactly as in one_tile, so the
-    // result is bit-identical.
-    auto two_tiles = [&](int k) -> bool {
-        const uint32_t sla = slot_of(k), slb = slot_of(k + 1);
-        if (!mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1)) return false;
-        if (!mbar_wait(bar0 + 8 * ((k + 1) % kStages), ((k + 1) / kStages) & 1)) return false;
-        const int tba = tile_base(k), tbb = tile_base(k + 1);
-        if (a.k_new != nullptr && tba + kTileTokens >= T) splice_new(k, tba);
-        if (a.k_new != nullptr && tbb + kTileTokens >= T) splice_new(k + 1, tbb);
-        clear_tail_v(k, tba);
-        clear_tail_v(k + 1, tbb);
-
-        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
-        float ta[4] = {0.f, 0.f, 0.f, 0.f}, tb[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int ks = 0; ks < 8; ks += 2) {
-            qk_step(sla, ks, sa);
-            qk_step(slb, ks, ta);
-            qk_step(sla, ks + 1, sb);
-            qk_step(slb, ks + 1, tb);
+    // Consecutive tiles of a warp feed different accumulators (kA = 2), so
+    // the second tile's work does not wait for the first tile's products.
+    for (int k = 0; k < my_tiles; k += kA) {
+        if (!one_tile(k, acc_state[0])) {
+            fail_k = k;
+            break;
         }
-        float xa[4], xb[4];
-        logits(sa, sb, tba, xa);
-        logits(ta, tb, tbb, xb);
-        float ma0 = fmaxf(xa[0], xa[2]), ma1 = fmaxf(xa[1], xa[3]);
-        float mb0 = fmaxf(xb[0], xb[2]), mb1 = fmaxf(xb[1], xb[3]);
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-            ma0 = fmaxf(ma0, __shfl_xor_sync(0xffffffffu, ma0, off));
-            ma1 = fmaxf(ma1, __shfl_xor_sync(0xffffffffu, ma1, off));
-            mb0 = fmaxf(mb0, __shfl_xor_sync(0xffffffffu, mb0, off));
-            mb1 = fmaxf(mb1, __shfl_xor_sync(0xffffffffu, mb1, off));
-        }
-        uint32_t pa01, pa23, pb01, pb23;
-        float ala0, ala1, alb0, alb1;
-        softmax_step(xa, ma0, ma1, pa01, pa23, ala0, ala1);
-        softmax_step(xb, mb0, mb1, pb01, pb23, alb0, alb1);
-        rescale(ala0, ala1);
-        const uint32_t pa0 = movmatrix_t(pa01), pa1 = movmatrix_t(pa23);
-        const uint32_t pb0 = movmatrix_t(pb01), pb1 = movmatrix_t(pb23);
-        uint32_t vb[8][4];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            uint32_t r0, r1, r2, r3;
-            const int u = 2 * i + vhi;
-            ldsm_x4_t(sla + 2 * kHalfBytes + (u >> 3) * kHalfBytes + swz(vrow, u & 7), r0, r1, r2,
-                      r3);
-            mma_bf16(o[i], r0, r1, r2, r3, pa0, pa1);
-            ldsm_x4_t(slb + 2 * kHalfBytes + (u >> 3) * kHalfBytes + swz(vrow, u & 7), vb[i][0],
-                      vb[i][1], vb[i][2], vb[i][3]);
-        }
-        rescale(alb0, alb1);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mma_bf16(o[i], vb[i][0], vb[i][1], vb[i][2], vb[i][3], pb0, pb1);
-        __syncwarp();
-        const int nblk0 = blk_of(k + kStages), nblk1 = blk_of(k + 1 + kStages);
-        if (lane == 0) {
-            if (k + kStages < my_tiles) issue(k + kStages, nblk0);
-            if (k + 1 + kStages < my_tiles) issue(k + 1 + kStages, nblk1);
-        }
-        return true;
-    };
-
-    for (int k = 0; k < my_tiles;) {
-        if (kStages == kStagesOne && k + 1 < my_tiles) {
-            if (!two_tiles(k)) {
-                fail_k = k;
+        if constexpr (kA == 2) {
+            if (k + 1 < my_tiles && !one_tile(k + 1, acc_state[1])) {
+                fail_k = k + 1;
                 break;
             }
-            k += 2;
-        } else {
-            if (!one_tile(k)) {
-                fail_k = k;
-                break;
-            }
-            k += 1;
         }
     }
 
@@ -517,60 +459,64 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
             mbar_wait(bar0 + 8 * (k % kStages), (k / kStages) & 1);
     }
 
-    // Normaliser: reduce the per-lane shares over the 8 lanes of a column.
-#pragma unroll
-    for (int off = 4; off < 32; off <<= 1) {
-        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-    }
-
-    // Warp state -> own ring (all of its loads have completed).
+    // Accumulator states -> this warp's own ring (all of its loads have
+    // completed): accumulator v = warp + kWarps * i at float offset
+    // i * kAccFloats of warp (v % kWarps)'s ring.
     constexpr int kOStride = kHeadDim + 4;   // floats per head row (bank skew)
-    float *ws = reinterpret_cast<float *>(ring);
-    float *wm = ws + kMaxGroup * kOStride;   // m[8], l[8]
-    {
+    constexpr int kAccFloats = kMaxGroup * kOStride + 2 * kMaxGroup;   // O rows, m[8], l[8]
+    static_assert(kA * kAccFloats * 4 <= kStages * kTileBytes, "states fit the ring");
+#pragma unroll
+    for (int i = 0; i < kA; ++i) {
+        AccState &s = acc_state[i];
+        // Normaliser: reduce the per-lane shares over the 8 lanes of a column.
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            s.l0 += __shfl_xor_sync(0xffffffffu, s.l0, off);
+            s.l1 += __shfl_xor_sync(0xffffffffu, s.l1, off);
+        }
+        float *ws = reinterpret_cast<float *>(ring) + i * kAccFloats;
+        float *wm = ws + kMaxGroup * kOStride;   // m[8], l[8]
         const int h0 = 2 * (lane & 3);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int d = 16 * i + (lane >> 2);
-            ws[h0 * kOStride + d] = o[i][0];
-            ws[(h0 + 1) * kOStride + d] = o[i][1];
-            ws[h0 * kOStride + d + 8] = o[i][2];
-            ws[(h0 + 1) * kOStride + d + 8] = o[i][3];
+        for (int r = 0; r < 8; ++r) {
+            const int d = 16 * r + (lane >> 2);
+            ws[h0 * kOStride + d] = s.o[r][0];
+            ws[(h0 + 1) * kOStride + d] = s.o[r][1];
+            ws[h0 * kOStride + d + 8] = s.o[r][2];
+            ws[(h0 + 1) * kOStride + d + 8] = s.o[r][3];
         }
         if (lane < 4) {
-            wm[h0] = m0;
-            wm[h0 + 1] = m1;
-            wm[8 + h0] = l0;
-            wm[8 + h0 + 1] = l1;
+            wm[h0] = s.m0;
+            wm[h0 + 1] = s.m1;
+            wm[8 + h0] = s.l0;
+            wm[8 + h0 + 1] = s.l1;
         }
     }
     __syncthreads();
 
-    // Merge warps in fixed order; thread handles (head, 8 dims).
+    // Merge the accumulators in order; a thread handles (head, 8 dims).
+    auto acc_base = [&](int v) {
+        return reinterpret_cast<const float *>(smem + (v % kWarps) * kStages * kTileBytes) +
+               (v / kWarps) * kAccFloats;
+    };
     const int64_t row_base = static_cast<int64_t>(lb) * sh.Hq + g * G;
     for (int e = threadIdx.x; e < G * (kHeadDim / 8); e += blockDim.x) {
         const int h = e / (kHeadDim / 8);
         const int d0 = (e % (kHeadDim / 8)) * 8;
         float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < kDecodeWarps; ++w) {
-            const float *wmw =
-                reinterpret_cast<const float *>(smem + w * kStages * kTileBytes) +
-                kMaxGroup * kOStride;
-            M = fmaxf(M, wmw[h]);
-        }
+        for (int v = 0; v < kAccs; ++v) M = fmaxf(M, acc_base(v)[kMaxGroup * kOStride + h]);
         float lsum = 0.f, acc[8];
 #pragma unroll
         for (int c = 0; c < 8; ++c) acc[c] = 0.f;
 #pragma unroll
-        for (int w = 0; w < kDecodeWarps; ++w) {
-            const float *wsw = reinterpret_cast<const float *>(smem + w * kStages * kTileBytes);
-            const float *wmw = wsw + kMaxGroup * kOStride;
-            const float sc = ex2(wmw[h] - M);
-            lsum += sc * wmw[8 + h];
+        for (int v = 0; v < kAccs; ++v) {
+            const float *wsv = acc_base(v);
+            const float *wmv = wsv + kMaxGroup * kOStride;
+            const float sc = ex2(wmv[h] - M);      // an accumulator with no tile: m = -inf, 0
+            lsum += sc * wmv[8 + h];
 #pragma unroll
-            for (int c = 0; c < 8; ++c) acc[c] += sc * wsw[h * kOStride + d0 + c];
+            for (int c = 0; c < 8; ++c) acc[c] += sc * wsv[h * kOStride + d0 + c];
         }
         if (nsplit == 1) {
             const float inv = 1.f / lsum;
@@ -716,17 +662,17 @@ bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const
 }
 
 cudaError_t prepare_kernels() {
-    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<kStagesFull>,
+    cudaError_t e = cudaFuncSetAttribute(decode_split_kernel<kWarpsNarrow, kStagesFull>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         decode_smem(kStagesFull));
+                                         decode_smem(kWarpsNarrow, kStagesFull));
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(decode_split_kernel<kStagesHalf>,
+        e = cudaFuncSetAttribute(decode_split_kernel<kWarpsNarrow, kStagesHalf>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 decode_smem(kStagesHalf));
+                                 decode_smem(kWarpsNarrow, kStagesHalf));
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(decode_split_kernel<kStagesOne>,
+        e = cudaFuncSetAttribute(decode_split_kernel<kWarpsWide, kStagesOne>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 decode_smem(kStagesOne));
+                                 decode_smem(kWarpsWide, kStagesOne));
     return e;
 }
 
@@ -741,7 +687,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
 
     cudaLaunchConfig_t c1 = {};
     c1.gridDim = dim3(splits, a.s.Hkv, a.nlayers * a.B);
-    c1.blockDim = dim3(kDecodeWarps * 32);
+    c1.blockDim = dim3(kWarpsNarrow * 32);
     c1.stream = st;
     c1.attrs = overlap_previous ? attr : nullptr;
     c1.numAttrs = overlap_previous ? 1 : 0;
@@ -756,14 +702,15 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
     };
     cudaError_t e;
     if (ctas <= num_sms) {
-        c1.dynamicSmemBytes = decode_smem(kStagesOne);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesOne>, map, a);
+        c1.blockDim = dim3(kWarpsWide * 32);
+        c1.dynamicSmemBytes = decode_smem(kWarpsWide, kStagesOne);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsWide, kStagesOne>, map, a);
     } else if (ctas <= 2 * static_cast<int64_t>(num_sms) || fill(2) > fill(3) + KVT_WAVE_MARGIN) {
-        c1.dynamicSmemBytes = decode_smem(kStagesHalf);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesHalf>, map, a);
+        c1.dynamicSmemBytes = decode_smem(kWarpsNarrow, kStagesHalf);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesHalf>, map, a);
     } else {
-        c1.dynamicSmemBytes = decode_smem(kStagesFull);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kStagesFull>, map, a);
+        c1.dynamicSmemBytes = decode_smem(kWarpsNarrow, kStagesFull);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesFull>, map, a);
     }
     if (e != cudaSuccess) return e;
     // Tables at most 1 024 tokens wide: every session is one split and the

@@ -164,10 +164,11 @@ def test_fused_steps_cross_blocks_and_splits(pkg):
 
 def test_fused_steps_one_cta_per_sm(pkg):
     """A batch small enough for one CTA per SM (3 splits x 4 kv-heads x 3
-    sessions = 36 CTAs) runs the kernel whose warps take their tiles in
-    pairs. Over twenty steps the token that arrives with the call lands in
-    the second tile of a pair and in a warp's lone last tile; the fused run
-    stays bit-identical to append-then-decode and agrees with the oracle."""
+    sessions = 36 CTAs) runs the 8-warp kernel, one accumulator per warp,
+    while larger grids run 4 warps with two accumulators each. Over twenty
+    steps the token that arrives with the call lands in different warps and
+    accumulators; the fused run stays bit-identical to append-then-decode
+    and agrees with the oracle."""
     lens = [70, 1100, 2030]
     pf, sids, T, of, q = run(pkg, True, lens, 20, L=2, mode="layer")
     pu, _, _, ou, _ = run(pkg, False, lens, 20, L=2, mode="layer")

@@ -140,19 +140,26 @@ def test_decode_independent_of_batch_and_placement(pkg):
 
 
 def test_ring_depths_bit_identical(pkg):
-    """The split kernel's tile-ring depth follows the size of the grid (6, 3
-    or 2 tiles in flight per warp for 1, 2 or 3 CTAs per SM). It changes only
-    how far ahead tiles are fetched, so all three must give the same bits."""
+    """The split kernel's launch variant follows the size of the grid: one
+    CTA per SM with 8 warps (one of a split's eight accumulators each), or 2
+    or 3 CTAs per SM with 4 warps (two accumulators each) and 3- or 2-deep
+    tile rings. The variants change where the accumulators run and how far
+    ahead tiles are fetched, never which tiles an accumulator takes or the
+    merge order, so all must give the same bits."""
     lens = [5000, 3001, 777]
     L = 16
     pool, sess, tables, q = direct_case(pkg, lens, L=L, seed=4, max_batch=L * len(lens))
+    mid = np.pad(tables, ((0, 0), (0, 600 - tables.shape[1])), constant_values=-1)
     wide = np.pad(tables, ((0, 0), (0, 2048 - tables.shape[1])), constant_values=-1)
-    # per layer, 313-block tables: 5 splits x 4 kv-heads x 3 rows = 60 CTAs (6-deep rings);
-    # per layer, tables 2048 blocks wide: 16 x 4 x 3 = 192 CTAs (3-deep);
-    # all 16 layers in one call: 5 x 4 x 48 = 960 CTAs (2-deep)
+    # per layer, 313-block tables: 5 splits x 4 kv-heads x 3 rows = 60 CTAs (8 warps);
+    # per layer, 600-block tables: 10 x 4 x 3 = 120 CTAs (8 warps);
+    # per layer, tables 2048 blocks wide: 16 x 4 x 3 = 192 CTAs (4 warps, 3-deep);
+    # all 16 layers in one call: 5 x 4 x 48 = 960 CTAs (4 warps, 2-deep)
     narrow = np.concatenate([gpu_decode(pool, l, q, tables, lens) for l in range(L)])
+    middle = np.concatenate([gpu_decode(pool, l, q, mid, lens) for l in range(L)])
     padded = np.concatenate([gpu_decode(pool, l, q, wide, lens) for l in range(L)])
     whole = gpu_decode(pool, -1, q, tables, lens)
+    assert np.array_equal(narrow.view(np.int64), middle.view(np.int64))
     assert np.array_equal(narrow.view(np.int64), padded.view(np.int64))
     assert np.array_equal(narrow.view(np.int64), whole.view(np.int64))
     ref = oracle.paged_decode(host_hot(pool, 4, sess, lens, tables), q.cpu().view(torch.int16)
