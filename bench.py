@@ -269,6 +269,11 @@ def run_decode(args, ws, rank):
         upload(0)
         for k in range(nsteps):
             buf = k % 2
+            if k >= 2:
+                # the host consumes step k-2's result before issuing step k, as a
+                # serving loop would; a host running further ahead fills the CUDA
+                # launch queue, where a launch waiting for room can stall it
+                down_done[buf].synchronize()
             if k + 1 < nsteps:
                 upload(buf ^ 1)
             stream.wait_event(up_done[buf])
@@ -559,6 +564,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
         "pauses_admissions_ms": round((h[1] - h[0]) * 1e3, 3),
         "reserve_ms": round(((h[2] or h[1]) - h[1]) * 1e3, 3),
         "decode_enqueue_ms": round((h[3] - (h[2] or h[1])) * 1e3, 3),
+        "thread_cpu_ms": round(h[4] * 1e3, 3),
         "gpu_ms": round(step_t[d.step_index.index(hk)][0], 3) if hk in d.step_index else None}
     if worst is not None:
         k = d.step_index[worst]
@@ -892,7 +898,7 @@ def main():
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--only-trace", action="store_true",
                     help="run only the agentic trace (simple and residency modes)")
-    ap.add_argument("--trace-max-ahead", type=int, default=3,
+    ap.add_argument("--trace-max-ahead", type=int, default=6,
                     help="trace: steps the host may run ahead of the GPU (0: unbounded)")
     ap.add_argument("--trace-no-overlap", action="store_true",
                     help="trace: launch every layer's decode fully serialised")

@@ -56,10 +56,11 @@ class TraceConfig:
     prefetch: bool = True            # residency mode: next step's spilled blocks fetched ahead
     overlap: bool = True             # layer l > 0 starts while layer l-1's call drains
     # The host issues step k only after step k - max_ahead has finished on the
-    # GPU (as a serving loop that reads back a step's tokens would); 0: never
-    # waits. A host that runs further ahead fills the CUDA launch queue, and a
-    # launch that waits for queue space can stall the host for tens of ms.
-    max_ahead: int = 3
+    # GPU; 0: never waits. The queued steps absorb host stalls (a descheduled
+    # thread on a shared machine); a host that runs further ahead than about
+    # ten steps fills the CUDA launch queue (about 1 000 launches), and a
+    # launch that waits for queue space can itself stall the host.
+    max_ahead: int = 6
 
 
 @dataclass
@@ -128,7 +129,8 @@ class TraceDriver:
         self.step_index = []                 # trace step k of each step_events entry
         self.mig_events = []                 # (kind, start, end, bytes)
         # host clock (perf_counter) per trace step: begin, after pauses and
-        # admissions, after the batch reservation, end of enqueue
+        # admissions, after the batch reservation, end of enqueue; then the
+        # CPU time the thread used over the step (time.thread_time)
         self.host_stamps = []
         self.gc_pauses = []                  # (generation, start, seconds) during run()
         self.admit_ev = {}
@@ -182,6 +184,7 @@ class TraceDriver:
         if self.gpu and cfg.max_ahead > 0 and len(self.step_events) >= cfg.max_ahead:
             self.step_events[-cfg.max_ahead][1].synchronize()
         h0 = time.perf_counter()
+        c0 = time.thread_time()
         h_adm = h_res = None
         now = k * cfg.dt_s
         tok_bytes = cfg.layers * 2 * cfg.num_kv_heads * 128 * 2
@@ -297,7 +300,7 @@ class TraceDriver:
                 self._prefetch_next(k, sids)
         self.counts["steps"] += 1
         self.counts["session_tokens"] += sum(self.tokens)
-        self.host_stamps.append((h0, h_adm, h_res, time.perf_counter()))
+        self.host_stamps.append((h0, h_adm, h_res, time.perf_counter(), time.thread_time() - c0))
 
     def _prefetch_next(self, k: int, busy: list) -> None:
         """One step ahead (Section 3, "Eviction, resume and decode"): the
