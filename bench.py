@@ -525,10 +525,13 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     # decode/migration overlap (Section 3: eviction and resume run beside
     # decode): every interval on one device clock, relative to the first step
     overlap = None
-    if d.step_events and d.mig_events:
+    if d.step_events and any(n > 0 for *_, n in d.mig_events):
         ref = d.step_events[0][0]
         steps_iv = [(ref.elapsed_time(a), ref.elapsed_time(b), tok) for a, b, _, tok in d.step_events]
-        migs_iv = [(ref.elapsed_time(a), ref.elapsed_time(b)) for _, a, b, _ in d.mig_events]
+        # migrations that moved bytes (a residency-mode prefetch with nothing
+        # missing, or a pause that packs nothing, is an empty interval)
+        migs_iv = [(ref.elapsed_time(a), ref.elapsed_time(b)) for _, a, b, n in d.mig_events
+                   if n > 0]
         mig_ms = sum(max(0.0, e - s0) for s0, e in migs_iv)
         inside = 0.0
         j = 0
