@@ -95,12 +95,14 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
     return true;
 }
 
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                            uint32_t bar) {
+// One tile: the box (64 columns, 16 rows, 2 column halves, K and V) of the
+// hot pool's 4-D view, starting at K row `row`.
+__device__ __forceinline__ void tma_load_tile(uint32_t dst, const CUtensorMap *map, int row,
+                                              uint32_t bar) {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(row), "r"(0), "r"(0), "r"(bar)
         : "memory");
 }
 
@@ -258,17 +260,13 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
             blk = 0;
         }
         const int rowk = ((blk * sh.L + l) * 2 * sh.Hkv + g) * sh.bt + (tok - j * sh.bt);
-        const int rowv = rowk + chunk_rows;
         const uint32_t slot = ring_s + (k % kStages) * kTileBytes;
         const uint32_t bar = bar0 + 8 * (k % kStages);
         // inject_extra_tx (a test of the bounded wait, 0 in normal calls): this
         // one barrier then never completes its phase, although every copy lands.
         const bool injected = k == 0 && warp == 0 && split == 0 && g == 0 && lb == 0;
         mbar_expect_tx(bar, kTileBytes + (injected ? a.inject_extra_tx : 0));
-        tma_load_2d(slot, &map, 0, rowk, bar);
-        tma_load_2d(slot + kHalfBytes, &map, 64, rowk, bar);
-        tma_load_2d(slot + 2 * kHalfBytes, &map, 0, rowv, bar);
-        tma_load_2d(slot + 3 * kHalfBytes, &map, 64, rowv, bar);
+        tma_load_tile(slot, &map, rowk, bar);
     };
     // The block of tile k, for every lane (k < 32 wherever it is used).
     auto blk_of = [&](int k) { return __shfl_sync(0xffffffffu, lane_blk, k & 31); };
@@ -630,7 +628,8 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
 
 }  // namespace
 
-bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why) {
+bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, int64_t run_rows,
+                           const char **why) {
     // Resolved once; a function-local static is initialised exactly once even
     // when pools are created, or allocation-free decodes issued, on several
     // host threads at the same moment.
@@ -647,11 +646,16 @@ bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const
         *why = "cuTensorMapEncodeTiled entry point unavailable";
         return false;
     }
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kRowBytes)};
-    cuuint32_t box[2] = {64, kTileTokens};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, hot_base, dims, strides, box, estr,
+    // A 4-D view of the pool: (64 columns, row, column half, K|V) with byte
+    // strides (2, 256, 128, run_rows * 256). A tile is one box of it: 16 rows
+    // of both halves of K and of V, landing in shared memory as [K|V][half]
+    // [row][64] with the 128-byte swizzle, the layout the kernel reads.
+    cuuint64_t dims[4] = {64, static_cast<cuuint64_t>(rows), 2, 2};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(kRowBytes), 128,
+                             static_cast<cuuint64_t>(run_rows) * kRowBytes};
+    cuuint32_t box[4] = {64, kTileTokens, 2, 2};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, hot_base, dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {

@@ -155,7 +155,10 @@ struct GatherArgs {
 };
 
 // Host launchers (decode_kernels.cu, copy_kernels.cu). Each returns the launch's CUDA status.
-bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, const char **why);
+// The decode kernel's tensor map of the hot pool: rows of 128 bf16, and
+// run_rows (Hkv * bt) rows between a (block, layer) K run and its V run.
+bool encode_hot_tensor_map(CUtensorMap *map, void *hot_base, int64_t rows, int64_t run_rows,
+                           const char **why);
 cudaError_t prepare_kernels();  // per-device function attributes
 // overlap_previous: launch the split kernel as a programmatic dependent of the
 // previous kernel on the stream (see decode_attention_ex). num_sms sizes the

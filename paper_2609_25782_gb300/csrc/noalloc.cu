@@ -25,7 +25,7 @@ static __device__ __align__(256) unsigned char g_decode_scratch[KV_NOALLOC_SCRAT
 constexpr int kMapCache = 4;
 struct CachedMap {
     const void *base = nullptr;
-    int64_t rows = 0;
+    int64_t rows = 0, run_rows = 0;
     uint64_t last_use = 0;
     CUtensorMap map{};
 };
@@ -69,12 +69,12 @@ int setup_device(int dev, unsigned char **ptr, int *num_sms) {
 
 // The hot arena's tensor map for this device: from the cache, else encoded
 // and put in place of the least recently used entry.
-int device_tensor_map(int dev, void *hot_base, int64_t rows, CUtensorMap *out) {
+int device_tensor_map(int dev, void *hot_base, int64_t rows, int64_t run_rows, CUtensorMap *out) {
     std::lock_guard<std::mutex> lk(g_mu);
     DeviceScratch &d = g_dev[dev];
     CachedMap *victim = &d.maps[0];
     for (CachedMap &m : d.maps) {
-        if (m.base == hot_base && m.rows == rows) {
+        if (m.base == hot_base && m.rows == rows && m.run_rows == run_rows) {
             m.last_use = ++d.clock;
             *out = m.map;
             return KV_OK;
@@ -83,9 +83,10 @@ int device_tensor_map(int dev, void *hot_base, int64_t rows, CUtensorMap *out) {
     }
     const char *why = nullptr;
     CUtensorMap map;
-    if (!kvt::encode_hot_tensor_map(&map, hot_base, rows, &why)) return fail(KV_ERR_CUDA, why);
+    if (!kvt::encode_hot_tensor_map(&map, hot_base, rows, run_rows, &why)) return fail(KV_ERR_CUDA, why);
     victim->base = hot_base;
     victim->rows = rows;
+    victim->run_rows = run_rows;
     victim->map = map;
     victim->last_use = ++d.clock;
     *out = map;
@@ -152,7 +153,8 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     int rc = setup_device(c.device, &scratch, &num_sms);
     if (rc) return rc;
     CUtensorMap map;
-    rc = device_tensor_map(c.device, c.hot_base, rows, &map);
+    rc = device_tensor_map(c.device, c.hot_base, rows,
+                           static_cast<int64_t>(c.num_kv_heads) * c.block_tokens, &map);
     if (rc) return rc;
 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

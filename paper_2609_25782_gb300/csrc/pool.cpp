@@ -474,7 +474,8 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
             });
         if (rc) return bail(rc);
         const char *why = nullptr;
-        if (!kvt::encode_hot_tensor_map(&p->tmap, c.hot_base, rows, &why))
+        if (!kvt::encode_hot_tensor_map(&p->tmap, c.hot_base, rows,
+                                        static_cast<int64_t>(c.num_kv_heads) * c.block_tokens, &why))
             return bail(fail(KV_ERR_CUDA, why));
         if (cudaDeviceSynchronize() != cudaSuccess)
             return bail(fail(KV_ERR_CUDA, "device synchronise after pool set-up failed"));
