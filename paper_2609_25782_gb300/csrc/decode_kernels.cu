@@ -40,6 +40,9 @@ constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
 // Each SM keeps about 24 tiles in flight whatever the variant, and every
 // variant gives bit-identical results.
 constexpr int kAccs = 8;
+// Lazy softmax maximum: the reference moves when a logit exceeds it by more
+// than this many powers of two (P then stays at most 2^8 = 256).
+constexpr float kLazyLog2 = 8.f;
 #ifndef KVT_WAVE_MARGIN
 #define KVT_WAVE_MARGIN 0.1   // last-wave fill gain that moves a grid to 2 CTAs per SM
 #endif
@@ -393,30 +396,43 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
         }
         float x[4];
         logits(sa, sb, tok_base, x);
-        float mx0 = fmaxf(x[0], x[2]), mx1 = fmaxf(x[1], x[3]);
+        // Online-softmax step with a lazy maximum: the reference point m moves
+        // only when a logit of the tile exceeds it by more than kLazyLog2 (the
+        // first tile always does, m starting at -inf); otherwise P = 2^(x - m)
+        // stays at most 2^kLazyLog2 and neither m, l nor the accumulator are
+        // rescaled. When it moves, m becomes the exact running maximum (a
+        // quad-shuffle reduction over the tile's columns) and l and O are
+        // rescaled by 2^(m_old - m_new). P is rounded to bf16, as the PV
+        // product sees it. The decision is the warp's and depends only on the
+        // tile's logits and the state, so every launch variant takes it alike.
+        const bool grow = (x[0] > s.m0 + kLazyLog2) | (x[2] > s.m0 + kLazyLog2) |
+                          (x[1] > s.m1 + kLazyLog2) | (x[3] > s.m1 + kLazyLog2);
+        if (__any_sync(0xffffffffu, grow)) {
+            float mx0 = fmaxf(x[0], x[2]), mx1 = fmaxf(x[1], x[3]);
 #pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+            for (int off = 4; off < 32; off <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+            }
+            const float mn0 = fmaxf(s.m0, mx0), mn1 = fmaxf(s.m1, mx1);
+            const float al0 = ex2(s.m0 - mn0), al1 = ex2(s.m1 - mn1);
+            s.m0 = mn0;
+            s.m1 = mn1;
+            s.l0 *= al0;
+            s.l1 *= al1;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                s.o[i][0] *= al0;
+                s.o[i][1] *= al1;
+                s.o[i][2] *= al0;
+                s.o[i][3] *= al1;
+            }
         }
-        // Online-softmax step: advance m and l, P rounded to bf16 (as the PV
-        // product sees it), the accumulator rescaled.
-        const float mn0 = fmaxf(s.m0, mx0), mn1 = fmaxf(s.m1, mx1);
-        const float al0 = ex2(s.m0 - mn0), al1 = ex2(s.m1 - mn1);
-        s.m0 = mn0;
-        s.m1 = mn1;
         float q0, q1, q2, q3;
-        const uint32_t p01 = pack_bf16(ex2(x[0] - mn0), ex2(x[1] - mn1), q0, q1);
-        const uint32_t p23 = pack_bf16(ex2(x[2] - mn0), ex2(x[3] - mn1), q2, q3);
-        s.l0 = s.l0 * al0 + q0 + q2;
-        s.l1 = s.l1 * al1 + q1 + q3;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            s.o[i][0] *= al0;
-            s.o[i][1] *= al1;
-            s.o[i][2] *= al0;
-            s.o[i][3] *= al1;
-        }
+        const uint32_t p01 = pack_bf16(ex2(x[0] - s.m0), ex2(x[1] - s.m1), q0, q1);
+        const uint32_t p23 = pack_bf16(ex2(x[2] - s.m0), ex2(x[3] - s.m1), q2, q3);
+        s.l0 += q0 + q2;
+        s.l1 += q1 + q3;
         const uint32_t pb0 = movmatrix_t(p01);   // P^T tokens 0-7  -> B fragment
         const uint32_t pb1 = movmatrix_t(p23);   // P^T tokens 8-15
         clear_tail_v(k, tok_base);
