@@ -459,7 +459,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
                          admit_lead=args.trace_admit_lead,
                          fused_append=not args.trace_unfused_append,
                          prefetch=not args.trace_no_prefetch,
-                         overlap=not args.trace_no_overlap, max_ahead=args.trace_max_ahead)
+                         overlap=not args.trace_no_overlap, max_ahead=args.trace_max_ahead,
+                         graphs=not args.trace_no_graphs)
     trace = tr.generate(cfg)
     plan = tr.plan(cfg, trace)
     nb = plan["peak_blocks"] + 256
@@ -615,6 +616,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     return {
         **extra,
         "admit_lead": cfg.admit_lead, "mig_ctas": args.trace_mig_ctas,
+        "decode_graphs": len(d.graphs) if cfg.graphs else None, "max_ahead": cfg.max_ahead,
         "step_append": "fused into the decode kernel" if cfg.fused_append else "separate kernel",
         "steps": cfg.steps, "sessions": cfg.sessions, "active_cap": cfg.active_cap,
         "step_ms_p50": round(pct(50), 3), "step_ms_p99": round(pct(99), 3),
@@ -901,8 +903,10 @@ def main():
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--only-trace", action="store_true",
                     help="run only the agentic trace (simple and residency modes)")
-    ap.add_argument("--trace-max-ahead", type=int, default=6,
+    ap.add_argument("--trace-max-ahead", type=int, default=20,
                     help="trace: steps the host may run ahead of the GPU (0: unbounded)")
+    ap.add_argument("--trace-no-graphs", action="store_true",
+                    help="trace: launch each step's decode calls directly (no CUDA graphs)")
     ap.add_argument("--trace-no-overlap", action="store_true",
                     help="trace: launch every layer's decode fully serialised")
     ap.add_argument("--trace-no-prefetch", action="store_true",

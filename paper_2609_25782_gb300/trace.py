@@ -55,12 +55,17 @@ class TraceConfig:
     fused_append: bool = True        # step token written by the decode kernel itself
     prefetch: bool = True            # residency mode: next step's spilled blocks fetched ahead
     overlap: bool = True             # layer l > 0 starts while layer l-1's call drains
+    # Each step's per-layer decode calls replayed from a CUDA graph, one per
+    # (batch size, table width rounded up to 1 024 tokens), as a serving
+    # engine replays decode graphs per batch bucket; the step's new K/V go
+    # through a fixed staging buffer.
+    graphs: bool = True
     # The host issues step k only after step k - max_ahead has finished on the
     # GPU; 0: never waits. The queued steps absorb host stalls (a descheduled
-    # thread on a shared machine); a host that runs further ahead than about
-    # ten steps fills the CUDA launch queue (about 1 000 launches), and a
-    # launch that waits for queue space can itself stall the host.
-    max_ahead: int = 6
+    # thread on a shared machine). The CUDA launch queue holds about 1 000
+    # launches (about ten steps of direct calls, about thirty replayed steps);
+    # a launch that waits for queue space can itself stall the host.
+    max_ahead: int = 20
 
 
 @dataclass
@@ -135,9 +140,15 @@ class TraceDriver:
         self.gc_pauses = []                  # (generation, start, seconds) during run()
         self.admit_ev = {}
         self.last_decode_ev = None
+        self.graphs = {}                     # (B, table width) -> captured decode step
         if gpu:
             import torch
             self._torch = torch
+            if cfg.graphs and cfg.fused_append:
+                shape = (cfg.layers, cfg.active_cap, cfg.num_kv_heads, 128)
+                dev = q.device
+                self.k_stage = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+                self.v_stage = torch.empty(shape, dtype=torch.bfloat16, device=dev)
 
     # ---------------------------------------------------------------- helpers
     def _event(self):
@@ -244,8 +255,12 @@ class TraceDriver:
             sids = [self.sids[i] for i in members]
             B = len(sids)
             # tables as wide as this batch's longest session (after its step token):
-            # no launched split lies past every session's end
+            # no launched split lies past every session's end; with graphs, rounded
+            # up to 1 024 tokens so that a step's graph is reused
             mb = -(-(max(self.tokens[i] for i in members) + 1) // cfg.block_tokens)
+            if self.gpu and cfg.graphs and self.max_blocks:
+                r = max(1, 1024 // cfg.block_tokens)
+                mb = min(self.max_blocks, -(-mb // r) * r)
             if cfg.fused_append:             # this step's token (path 3) comes with the decode
                 if self.gpu:
                     with self._torch.cuda.stream(self.dstream):
@@ -271,20 +286,24 @@ class TraceDriver:
                          for i in self.active + [i for _, i in self.joining])
             self.peak_blocks = max(self.peak_blocks, blocks)
             if self.gpu:
-                for l in range(cfg.layers):
-                    # layer l > 0 follows layer l-1's call, which writes only `out`
-                    # and (fused) layer l-1's rows of the pool
-                    flags = kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 and cfg.overlap else 0
-                    if cfg.fused_append:
-                        kvtier.decode_append_attention(
-                            self.pool, l, self.q[l], k_new[l], v_new[l], self.tables,
-                            self.seq_lens, B, mb, 1 / math.sqrt(128), self.out[l],
-                            flags, self.dstream)
-                    else:
-                        kvtier.decode_attention_ex(
-                            self.pool, l, self.q[l], self.tables, self.seq_lens, B,
-                            mb, 1 / math.sqrt(128), self.out[l], flags,
-                            self.dstream)
+                if cfg.fused_append and cfg.graphs:
+                    with self._torch.cuda.stream(self.dstream):   # fixed addresses
+                        self.k_stage[:, :B].copy_(k_new)
+                        self.v_stage[:, :B].copy_(v_new)
+                    k_new, v_new = self.k_stage, self.v_stage
+                g = self.graphs.get((B, mb)) if cfg.graphs else None
+                if g is not None:
+                    with self._torch.cuda.stream(self.dstream):
+                        g.replay()
+                else:
+                    self._decode_calls(B, mb, k_new, v_new)
+                    if cfg.graphs:               # record it for the next step of this shape
+                        g = self._torch.cuda.CUDAGraph()
+                        with self._torch.cuda.stream(self.dstream):
+                            g.capture_begin(capture_error_mode="relaxed")
+                            self._decode_calls(B, mb, k_new, v_new)
+                            g.capture_end()
+                        self.graphs[(B, mb)] = g
                 end.record(self.dstream)
                 self.last_decode_ev = end
                 self.step_events.append((start, end, B, sum(self.tokens[i] for i in members)))
@@ -301,6 +320,22 @@ class TraceDriver:
         self.counts["steps"] += 1
         self.counts["session_tokens"] += sum(self.tokens)
         self.host_stamps.append((h0, h_adm, h_res, time.perf_counter(), time.thread_time() - c0))
+
+    def _decode_calls(self, B: int, mb: int, k_new, v_new) -> None:
+        """The step's per-layer decode calls on the decode stream."""
+        cfg = self.cfg
+        for l in range(cfg.layers):
+            # layer l > 0 follows layer l-1's call, which writes only `out`
+            # and (fused) layer l-1's rows of the pool
+            flags = kvtier.KV_DECODE_OVERLAP_PREVIOUS if l > 0 and cfg.overlap else 0
+            if cfg.fused_append:
+                kvtier.decode_append_attention(
+                    self.pool, l, self.q[l], k_new[l], v_new[l], self.tables, self.seq_lens, B,
+                    mb, 1 / math.sqrt(128), self.out[l], flags, self.dstream)
+            else:
+                kvtier.decode_attention_ex(
+                    self.pool, l, self.q[l], self.tables, self.seq_lens, B, mb,
+                    1 / math.sqrt(128), self.out[l], flags, self.dstream)
 
     def _prefetch_next(self, k: int, busy: list) -> None:
         """One step ahead (Section 3, "Eviction, resume and decode"): the

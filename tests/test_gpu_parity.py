@@ -557,3 +557,35 @@ def test_decode_extreme_logits(pkg, case):
             for g in range(4):
                 assert np.allclose(got[0, b, g * 8], v[g], rtol=1e-5, atol=1e-6)
     assert pool.check_device() == 0
+
+
+def test_device_table_row_matches_host_row(pkg):
+    """session_block_table_device: the address of a session's row in the
+    pool's device table arena, fixed for the pool's life; after appends and
+    after a pause and a resume into other blocks it holds the same ids as
+    the host copy (read here through the CUDA array interface)."""
+    dev = torch.device("cuda:0")
+    pool = pkg.Pool(num_layers=2, num_hot_blocks=64, cold_bytes=1 << 24, max_sessions=2,
+                    max_batch=4, max_context=512, alloc_seed=5)
+    s = pool.session_create(512)
+    k, v = synth.kv_logical_torch(1, s, range(2), 4, 128, 0, 300, dev)
+    pool.session_append(s, k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous())
+    addr, n = pool.session_block_table_device(s)
+    assert n == len(pool.session_block_table(s)) == -(-300 // 16)
+
+    class Row:
+        __cuda_array_interface__ = {"shape": (n,), "typestr": "<i4", "data": (addr, False),
+                                    "version": 2}
+
+    row = torch.as_tensor(Row(), device=dev)
+    torch.cuda.synchronize()
+    assert row.cpu().tolist() == pool.session_block_table(s)
+    old = pool.session_block_table(s)
+    pool.session_pause(s)
+    pool.shuffle_free(9)
+    pool.session_resume(s)
+    torch.cuda.synchronize()
+    assert pool.session_block_table_device(s) == (addr, n)
+    assert row.cpu().tolist() == pool.session_block_table(s) != old
+    assert pool.check_device() == 0
+    pool.close()
