@@ -253,3 +253,67 @@ def test_small_trace_residency_under_pressure(cuda_dev, prefetch, lead):
                 "blocks_prefetched", "prefetches"):
         assert st[key] == dry[key], key
     pool.close()
+
+
+def test_trace_graph_replay_bit_identical_to_direct_calls(cuda_dev):
+    """The driver replays each step's per-layer calls from a CUDA graph cached
+    per (batch size, table width rounded up to 1 024 tokens), the step's new
+    K/V staged in a fixed buffer. On the same schedule the outputs of every
+    step must be bit-identical to launching the calls directly (the wider
+    tables change the launch shape only)."""
+    import dataclasses
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool
+    from paper_2609_25782_gb300 import trace as tr
+
+    base = tr.TraceConfig(sessions=6, t0_min=100, t0_max=1500, burst_mean=8.0, pause_mean_s=0.6,
+                          append_median=40.0, append_sigma=1.0, append_max=300, active_cap=3,
+                          steps=80, dt_s=0.1, layers=2, seed=7)
+    trace = tr.generate(base)
+    plan = tr.plan(base, trace)
+    L, Hkv, Hq, D, bt = base.layers, base.num_kv_heads, base.num_q_heads, 128, base.block_tokens
+    outs = {}
+    for graphs in (True, False):
+        cfg = dataclasses.replace(base, graphs=graphs)
+        pool = Pool(num_layers=L, num_hot_blocks=plan["peak_blocks"] + 40,
+                    cold_bytes=plan["cold_bytes"] + 4096, max_sessions=cfg.sessions,
+                    max_batch=cfg.active_cap, max_context=plan["max_context"], alloc_seed=3)
+        for i, t in enumerate(trace):
+            sid = pool.session_create_paused(plan["caps"][i], t.t0)
+            synth.fill_image_torch(pool.image(sid), cfg.seed, sid, L, Hkv, D, t.t0)
+
+        def kv_source(sid, t0, t1):
+            k, v = synth.kv_logical_torch(cfg.seed, sid, range(L), Hkv, D, t0, t1, cuda_dev)
+            return k.permute(0, 2, 1, 3).contiguous(), v.permute(0, 2, 1, 3).contiguous()
+
+        q = synth.queries_torch(cfg.seed, range(cfg.active_cap), range(L), Hq, D, cuda_dev)
+        out = torch.empty(L, cfg.active_cap, Hq, D, dtype=torch.float32, device=cuda_dev)
+        max_blocks = -(-plan["max_context"] // bt)
+        tables = torch.empty(cfg.active_cap, max_blocks, dtype=torch.int32, device=cuda_dev)
+        seq_lens = torch.empty(cfg.active_cap, dtype=torch.int32, device=cuda_dev)
+        torch.cuda.synchronize()
+        got = {}
+
+        def on_step(k, members, out=out, got=got):
+            torch.cuda.synchronize()
+            got[k] = (tuple(members), out[:, :len(members)].clone())
+
+        d = tr.TraceDriver(cfg, pool.handle, trace, gpu=True, kv_source=kv_source, q=q, out=out,
+                           decode_stream=torch.cuda.Stream(), mig_stream=torch.cuda.Stream(),
+                           tables=tables, seq_lens=seq_lens, max_blocks=max_blocks,
+                           on_step=on_step)
+        d.run()
+        torch.cuda.synchronize()
+        assert pool.check_device() == 0
+        if graphs:
+            assert 0 < len(d.graphs) < len(got)      # shapes repeat: graphs are replayed
+        outs[graphs] = got
+        pool.close()
+    assert outs[True].keys() == outs[False].keys() and len(outs[True]) > 40
+    for k in outs[True]:
+        mg, og = outs[True][k]
+        md, od = outs[False][k]
+        assert mg == md
+        assert torch.equal(og.view(torch.int32), od.view(torch.int32)), k
