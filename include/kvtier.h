@@ -84,7 +84,9 @@ enum { KV_SESSION_FREE = 0, KV_SESSION_ACTIVE = 1, KV_SESSION_PAUSED = 2 };
  *    (write-on-evict, Section 3, "Memory hierarchy and write policy");
  *  - session_resume fetches only the blocks that are no longer hot (the
  *    others count as resume hits), and kv_pool_batch_tables first fetches
- *    any evicted block of its sessions;
+ *    any evicted block of its sessions (kv_pool_prefetch fetches them one
+ *    step ahead); a fetch waits for the evictions that wrote the session's
+ *    image, whatever stream they ran on;
  *  - evicted slots go to the end of the free list, in eviction order, and the
  *    call's allocations pop from the end.
  * Any call that allocates may evict blocks of any other session, so order it
