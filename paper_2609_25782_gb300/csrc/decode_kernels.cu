@@ -10,9 +10,9 @@
 //                          kernel.
 //
 // Hot pool: hot[NB][L][2][Hkv][bt][128] bf16. A (block, layer, K|V, head)
-// run is bt rows of 256 B. The decode kernel views the pool as a 2-D tensor
-// of 128-element rows (row = ((blk*L + l)*2 + kv)*Hkv + g)*bt + slot) and
-// loads 16-row x 64-column boxes.
+// run is bt rows of 256 B, row = ((blk*L + l)*2 + kv)*Hkv + g)*bt + slot. The
+// decode kernel views the pool as a 4-D tensor (64 columns, row, column half,
+// K|V) and loads one box per 16-token tile: its 16 K rows and 16 V rows.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
