@@ -251,3 +251,88 @@ def test_fetch_waits_for_an_eviction_on_another_stream(cuda_dev):
         assert np.array_equal(hb[:, 0, :, :n], k[:, :, j * bt:j * bt + n])
         assert np.array_equal(hb[:, 1, :, :n], v[:, :, j * bt:j * bt + n])
     pool.close()
+
+
+def test_prefetch_beside_a_running_step(cuda_dev):
+    """kv_pool_prefetch as the trace driver uses it: while step k (sessions
+    A, B) is still queued on the decode stream behind a spin, the prefetch of
+    step k+1's sessions (C, two of whose blocks were evicted, and D) runs on
+    the migration stream, evicting only the idle session E. Both steps must
+    match the oracle, and step k+1 must find nothing left to fetch."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_25782_gb300 import Pool
+
+    L, Hq, Hkv, D, bt, seed, cap = 2, 32, 4, 128, 16, 41, 200
+    nb = 19                            # exactly the five sessions' blocks
+    pool = Pool(num_layers=L, num_hot_blocks=nb, cold_bytes=6 * cap * pool_token_bytes(L, Hkv),
+                max_sessions=6, max_batch=L * 2, max_context=cap, alloc_seed=seed,
+                lru_residency=True)
+    o = ResidencyOracle(nb, bt, seed=seed, token_bytes=pool.token_bytes)
+    dst, mst = torch.cuda.Stream(), torch.cuda.Stream()
+    T = {}
+
+    def create(n0):
+        sid = pool.session_create_paused(cap, n0)
+        with torch.cuda.stream(mst):
+            synth.fill_image_torch(pool.image(sid), seed, sid, L, Hkv, D, n0)
+        o.create_paused(sid, cap, n0)
+        T[sid] = n0
+        return sid
+
+    e, c, a, b, d = (create(n) for n in (96, 80, 48, 48, 32))
+    for sid in (c, e, a, b, d):        # C least recent, then E; the pool is full
+        pool.session_resume(sid, mst)
+        o.resume(sid)
+    k_, v_ = synth.kv_logical_torch(seed, d, range(L), Hkv, D, T[d], T[d] + 32, cuda_dev)
+    with torch.cuda.stream(mst):       # D grows by two blocks: C's blocks 0 and 1 go
+        pool.session_append(d, k_.permute(0, 2, 1, 3).contiguous(),
+                            v_.permute(0, 2, 1, 3).contiguous(), mst)
+    o.append(d, 32)
+    T[d] += 32
+    torch.cuda.synchronize()
+    assert o.row(c)[:2] == [-1, -1] and min(o.row(c)[2:]) >= 0
+
+    mb = -(-cap // bt)
+    tables = [torch.empty(2, mb, dtype=torch.int32, device=cuda_dev) for _ in range(2)]
+    slens = [torch.empty(2, dtype=torch.int32, device=cuda_dev) for _ in range(2)]
+    q = synth.queries_torch(seed, range(2), range(L), Hq, D, cuda_dev)
+    outs = []
+    torch.cuda.synchronize()
+
+    def step(i, batch, spin):
+        with torch.cuda.stream(dst):
+            if spin:
+                torch.cuda._sleep(100_000_000)   # hold the step back (about 50 ms)
+            pool.batch_tables(batch, tables[i], mb, slens[i], dst)
+            o.batch(batch)
+            out = torch.empty(L, 2, Hq, D, dtype=torch.float32, device=cuda_dev)
+            pool.decode_attention(-1, q, tables[i], slens[i], 2, mb, 1 / math.sqrt(D), out, dst)
+            done = torch.cuda.Event()
+            done.record(dst)
+        rows = np.full((2, mb), -1, dtype=np.int32)
+        for r, x in enumerate(batch):
+            rows[r, :len(o.row(x))] = o.row(x)
+        outs.append((out, rows, [T[x] for x in batch], batch))
+        return done
+
+    done_k = step(0, [a, b], spin=True)
+    pool.prefetch([c, d], busy=[a, b], stream=mst)   # beside step k; victims outside A-D
+    o.prefetch([c, d], [a, b])
+    assert o.stats["blocks_prefetched"] == 2 and o.row(e)[:2] == [-1, -1]
+    mst.wait_event(done_k)
+    fetched = o.stats["batch_blocks_fetched"]
+    step(1, [c, d], spin=False)
+    assert o.stats["batch_blocks_fetched"] == fetched   # nothing left for step k+1
+    torch.cuda.synchronize()
+    assert pool.check_device() == 0
+    for key in ("blocks_evicted", "bytes_packed", "bytes_unpacked", "blocks_prefetched",
+                "batch_blocks_fetched"):
+        assert pool.stats()[key] == o.stats[key], key
+    for out, rows, lens, batch in outs:
+        hot = synth.hot_pool_np(seed, batch, lens, rows, nb, L, Hkv, D, bt)
+        ref = oracle.paged_decode(hot, bits(q), rows, lens, 1 / math.sqrt(D), Hq)
+        got = out.double().cpu().numpy()
+        assert np.all(np.isfinite(got))
+        assert np.max(np.abs(got - ref) / np.maximum(1.0, np.abs(ref))) <= TOL
+    pool.close()
