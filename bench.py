@@ -303,9 +303,15 @@ def run_decode(args, ws, rank):
     if ws > 1:
         dist.barrier()
 
-    # the library launches the combine only when a session can have two splits
-    # (tables wider than 1 024 tokens)
-    per_call = 1 if max_blocks * BT <= 1024 else 2
+    # Launches per call, as the library decides them: the split kernel, plus
+    # the combine when a session of the table's width can have more splits
+    # than the split kernel merges itself (16 when the grid of splits x
+    # kv-heads x rows fits the SMs at once, else 4).
+    from paper_2609_25782_gb300 import kvtier
+    splits = kvtier.kv_decode_splits(max_blocks * BT)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    in_kernel = 16 if splits * HKV * B2 <= 2 * sms else 4
+    per_call = 1 if splits <= max(1, in_kernel) else 2
     res = {
         "graph": graph is not None, "launches_per_call": per_call,
         "total_ms": total_ms, "launch_ms": launch_ms, "kv_bytes": kv_bytes, "e2e_ms": e2e_ms,
@@ -560,7 +566,15 @@ def run_trace(args, rank, lru_factor: float = 0.0):
     host = {"enqueue_ms_p50": round(host_ms[len(host_ms) // 2], 3),
             "enqueue_ms_max": round(host_ms[-1], 3),
             "gc_pauses": len(d.gc_pauses),
-            "gc_pause_ms_max": round(max((p[2] for p in d.gc_pauses), default=0.0) * 1e3, 3)}
+            "gc_pause_ms_max": round(max((p[2] for p in d.gc_pauses), default=0.0) * 1e3, 3),
+            # decode steps queued on the GPU when the host began a step
+            "queued_steps_p50": sorted(h[5] for h in d.host_stamps)[len(d.host_stamps) // 2]}
+    # time the thread spent off the CPU inside a step (blocked in a call, or
+    # descheduled): wall time minus thread CPU time
+    off = sorted(max(0.0, (h[3] - h[0]) - h[4]) * 1e3 for h in d.host_stamps)
+    host["offcpu_ms_p99"] = round(off[int(0.99 * (len(off) - 1))], 3)
+    host["offcpu_ms_max"] = round(off[-1], 3)
+    host["steps_offcpu_over_1ms"] = sum(1 for x in off if x > 1.0)
     hk = max(range(len(d.host_stamps)), key=lambda i: d.host_stamps[i][3] - d.host_stamps[i][0])
     h = d.host_stamps[hk]
     host["slowest_host_step"] = {
@@ -569,6 +583,7 @@ def run_trace(args, rank, lru_factor: float = 0.0):
         "reserve_ms": round(((h[2] or h[1]) - h[1]) * 1e3, 3),
         "decode_enqueue_ms": round((h[3] - (h[2] or h[1])) * 1e3, 3),
         "thread_cpu_ms": round(h[4] * 1e3, 3),
+        "queued_steps_at_start": h[5],
         "gpu_ms": round(step_t[d.step_index.index(hk)][0], 3) if hk in d.step_index else None}
     if worst is not None:
         k = d.step_index[worst]
@@ -578,6 +593,8 @@ def run_trace(args, rank, lru_factor: float = 0.0):
             "step": k, "ms": round(step_t[worst][0], 3),
             "host_enqueue_ms": round((d.host_stamps[k][3] - d.host_stamps[k][0]) * 1e3, 3),
             "host_ms_prev8_max": round(max((h[3] - h[0]) * 1e3 for h in d.host_stamps[lo:k + 1]), 3),
+            "queued_steps_at_start": d.host_stamps[k][5],
+            "queued_steps_prev8_min": min(h[5] for h in d.host_stamps[lo:k + 1]),
             "gc_ms_in_prev8": round(sum(p[2] for p in d.gc_pauses
                                         if t_lo <= p[1] <= t_hi) * 1e3, 3)}
     torch.cuda.empty_cache()

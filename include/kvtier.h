@@ -226,7 +226,10 @@ int session_append(kv_pool *pool, int32_t sid, const void *k, const void *v, int
  * (ceil(t / 1024) up to 16 splits, ceil(t / 2048) beyond 32K tokens); a
  * call needs
  * layers x B x Hq x S(max_blocks x bt) rows, else KV_ERR_INVALID_ARG. Calls on
- * one pool share the workspace: issue them in order on one stream. */
+ * one pool share the workspace (the partials, and one split-arrival counter
+ * per (row, kv-head) that every call leaves at zero): issue them in order on
+ * one stream. Calls whose work overlaps on the GPU give wrong results, and
+ * counters they leave non-zero make later multi-split results wrong too. */
 int decode_attention(kv_pool *pool, int32_t layer, const void *q,
                      const int32_t *block_tables, const int32_t *seq_lens, int32_t B,
                      int32_t max_blocks, float scale, float *out, kv_stream_t stream);
@@ -438,9 +441,11 @@ int kv_pool_inject_decode_timeout(kv_pool *pool, int32_t on);
  * The first call on a device, with that device current, looks up the
  * array's device address (cudaGetSymbolAddress) and sets the decode
  * kernel's shared-memory attribute; make that first call before any stream
- * capture. All calls share the one array: calls whose work overlaps on the
+ * capture. All calls share the one array, and one array of split-arrival
+ * counters that every call leaves at zero: calls whose work overlaps on the
  * GPU (different streams, or different host threads without ordering) race
- * and give wrong results; order them on one stream. Kernel bounds checks
+ * and give wrong results, and counters they leave non-zero make later calls
+ * wrong too; order them on one stream. Kernel bounds checks
  * keep bad block ids or lengths memory-safe but are not reported here: a
  * row whose seq_len is below 1 or beyond max_blocks * block_tokens is not
  * written at all (out keeps what it held), a block id outside the pool is

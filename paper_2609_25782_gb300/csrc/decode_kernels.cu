@@ -5,9 +5,13 @@
 //                          staged by TMA (cp.async.bulk.tensor, 128-byte
 //                          swizzle) into a per-warp mbarrier ring, and the
 //                          group-by-tile products run on mma.sync bf16.
-//   decode_combine_kernel  log-sum-exp merge of the splits in a fixed order,
-//                          launched as a programmatic dependent of the split
-//                          kernel.
+//                          The last CTA of a session's kv-head to finish
+//                          merges its splits (log-sum-exp in a fixed order)
+//                          when they are few: up to 16 in a grid that fits
+//                          the SMs at once, up to 4 in a longer one.
+//   decode_combine_kernel  the same merge for the other multi-split
+//                          sessions, launched as a programmatic dependent of
+//                          the split kernel when the table width allows them.
 //
 // Hot pool: hot[NB][L][2][Hkv][bt][128] bf16. A (block, layer, K|V, head)
 // run is bt rows of 256 B, row = ((blk*L + l)*2 + kv)*Hkv + g)*bt + slot. The
@@ -25,6 +29,15 @@ namespace {
 #define KVT_STAGES 2   // 4 warps x 2 x 8 KiB: 3 CTAs (24 tiles in flight) per SM
 #endif
 constexpr int kCombineWarps = 4;
+// The merge of a session's splits folds four chains (contiguous quarters of
+// the splits, in split order) and then merges the chains in order; that order
+// depends on the split count only, whichever kernel runs it. The split
+// kernel's last CTA of a (row, kv-head) can take up to kMergeInKernel splits
+// (four per chain).
+constexpr int kMergeChains = 4;
+constexpr int kMergeInKernel = 16;
+static_assert(kCombineWarps == kMergeChains && kMergeInKernel == kMergeChains * 4,
+              "four splits per chain in the split kernel, one chain per combine warp");
 constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
 constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
 // The plan of one split: its tiles are dealt round robin to kAccs running
@@ -158,6 +171,110 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
     return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4));
 }
 
+// Acquire-release add at GPU scope: orders this CTA's partial writes (made
+// visible to thread 0 by the preceding barrier) before its arrival, and the
+// last arrival's reads of the other partials after it.
+__device__ __forceinline__ int arrive(int32_t *counter) {
+    int prev;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
+                 : "=r"(prev)
+                 : "l"(counter)
+                 : "memory");
+    return prev;
+}
+
+// One step of a running log-sum-exp merge: fold the partial (m, l) = v with
+// accumulator o into (m, lsum, acc). The roundings are spelled out (one
+// product, then one fused multiply-add), so that the split kernel and the
+// combine kernel, which both run this, give the same bits.
+__device__ __forceinline__ float fold(float x, float c, float w, float y) {
+    return __fmaf_rn(x, c, __fmul_rn(w, y));
+}
+__device__ __forceinline__ void lse_step(float &m, float &lsum, float4 &acc, const float2 v,
+                                         const float4 o) {
+    const float mn = fmaxf(m, v.x);
+    const float c = ex2(m - mn);                   // rescale what is summed so far
+    const float w = ex2(v.x - mn);
+    m = mn;
+    lsum = fold(lsum, c, w, v.y);
+    acc.x = fold(acc.x, c, w, o.x);
+    acc.y = fold(acc.y, c, w, o.y);
+    acc.z = fold(acc.z, c, w, o.z);
+    acc.w = fold(acc.w, c, w, o.w);
+}
+
+// The chains' states merged in chain order and normalised; lane t writes
+// dims 4t..4t+3 of output row `row`.
+__device__ __forceinline__ void merge_chains_store(const DecodeArgs &a, int64_t row, int lane,
+                                                   const float (&m)[kMergeChains],
+                                                   const float (&l)[kMergeChains],
+                                                   const float4 (&acc)[kMergeChains]) {
+    float M = m[0];
+#pragma unroll
+    for (int q = 1; q < kMergeChains; ++q) M = fmaxf(M, m[q]);
+    float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+    float lt = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMergeChains; ++q) {
+        const float c = ex2(m[q] - M);             // an empty chain has m = -inf: c = 0
+        r.x = __fmaf_rn(c, acc[q].x, r.x);
+        r.y = __fmaf_rn(c, acc[q].y, r.y);
+        r.z = __fmaf_rn(c, acc[q].z, r.z);
+        r.w = __fmaf_rn(c, acc[q].w, r.w);
+        lt = __fmaf_rn(c, l[q], lt);
+    }
+    const float inv = __frcp_rn(lt);
+    const float4 y = make_float4(__fmul_rn(r.x, inv), __fmul_rn(r.y, inv), __fmul_rn(r.z, inv),
+                                 __fmul_rn(r.w, inv));
+    if (a.out_bf16) {
+        float r0, r1;
+        uint2 pk;
+        pk.x = pack_bf16(y.x, y.y, r0, r1);
+        pk.y = pack_bf16(y.z, y.w, r0, r1);
+        reinterpret_cast<uint2 *>(reinterpret_cast<uint16_t *>(a.out) + row * kHeadDim)[lane] = pk;
+    } else {
+        reinterpret_cast<float4 *>(a.out + row * kHeadDim)[lane] = y;
+    }
+}
+
+// The merge of one query head's ns (2..16) split partials by one warp. Every
+// load is issued before the first is used (indices clamped into the row, so
+// the loads need no guard): lane t loads split t's (m, l), shared by shuffle,
+// and each lane its 4 dims of every split's accumulator. The partials come
+// from L2 (.cg), written there by other SMs.
+__device__ __forceinline__ void merge_head_in_kernel(const DecodeArgs &a, int64_t row, int ns,
+                                                     int lane) {
+    const int64_t base = row * a.max_splits;
+    const float2 mine = __ldcg(reinterpret_cast<const float2 *>(a.part_ml) + base +
+                               min(lane, ns - 1));
+    const float4 *po = reinterpret_cast<const float4 *>(a.part_o + base * kHeadDim) + lane;
+    float4 o[kMergeChains][4];
+    int s0[kMergeChains], n[kMergeChains];
+#pragma unroll
+    for (int q = 0; q < kMergeChains; ++q) {
+        s0[q] = (q * ns) / kMergeChains;
+        n[q] = ((q + 1) * ns) / kMergeChains - s0[q];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) o[q][i] = __ldcg(po + min(s0[q] + i, ns - 1) * (kHeadDim / 4));
+    }
+    float m[kMergeChains], l[kMergeChains];
+    float4 acc[kMergeChains];
+#pragma unroll
+    for (int q = 0; q < kMergeChains; ++q) {
+        m[q] = -INFINITY;
+        l[q] = 0.f;
+        acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int sp = min(s0[q] + i, ns - 1);
+            const float2 v = make_float2(__shfl_sync(0xffffffffu, mine.x, sp),
+                                         __shfl_sync(0xffffffffu, mine.y, sp));
+            if (i < n[q]) lse_step(m[q], l[q], acc[q], v, o[q][i]);
+        }
+    }
+    merge_chains_store(a, row, lane, m, l, acc);
+}
+
 // ---------------------------------------------------------------------------
 // K1: one CTA = (split s, kv-head g, layer-batch row lb = li*B + b).
 // The split's tiles go round robin to kAccs = 8 accumulators; warp w of the
@@ -168,7 +285,8 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 //   online softmax over tokens (columns = heads)
 //   O^T[128 x 8] += V^T[128 x 16] . P^T[16 x 8]     8 x mma, P^T via movmatrix
 // The accumulators merge in shared memory in accumulator order; a one-split
-// session writes its normalised output, others write (m, l, acc) partials.
+// session writes its normalised output, others write (m, l, acc) partials,
+// which the group's last CTA to finish merges when there are at most 16.
 // ---------------------------------------------------------------------------
 struct AccState {
     float m0, m1;   // running max, heads 2(lane%4) and +1 (log2 units)
@@ -203,8 +321,9 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
     const Shape sh = a.s;
     const int G = sh.Hq / sh.Hkv;
 
-    // The combine kernel may be scheduled once every CTA of this grid has
-    // started; it still waits for this grid to finish before reading.
+    // The combine kernel, or the next call launched with the overlap option,
+    // may be scheduled once every CTA of this grid has started; it still
+    // waits for this grid to finish before reading.
     asm volatile("griddepcontrol.launch_dependents;");
     const int32_t *trow = a.tables + static_cast<int64_t>(b) * a.max_blocks;
     // Tables at most KVT_SPLIT_TARGET x KVT_SPLIT_MIN_TILES tiles wide split
@@ -559,12 +678,30 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
             }
         }
     }
+    if (nsplit == 1 || nsplit > a.merge_max_splits) return;
+
+    // Arrival. Every split of the group arrives once, whatever happened in
+    // it; the last one merges the group's G heads (a warp per head) and
+    // resets the counter for the next call, which touches it only after this
+    // grid has completed.
+    __shared__ int s_last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int32_t *counter = a.counters + static_cast<int64_t>(lb) * sh.Hkv + g;
+        const bool last = arrive(counter) == nsplit - 1;
+        if (last) *counter = 0;
+        s_last = last;
+    }
+    __syncthreads();
+    if (!s_last) return;
+#pragma unroll 1
+    for (int h = warp; h < G; h += kWarps) merge_head_in_kernel(a, row_base + h, nsplit, lane);
 }
 
-// K2: one CTA (4 warps) per (layer-batch row, q-head) of a multi-split
-// session. Warp w merges the contiguous quarter [w*ns/4, (w+1)*ns/4) of the
-// splits with a running log-sum-exp (split order), then warp 0 merges the
-// four warp states in warp order. The result depends only on the partials
+// K2: one CTA (4 warps) per (layer-batch row, q-head) of a session of more
+// than kMergeInKernel splits. Warp w folds chain w, the contiguous quarter
+// [w*ns/4, (w+1)*ns/4) of the splits (split order), then warp 0 merges the
+// four chains in order. The result depends only on the partials
 // and ns. Launched as a programmatic dependent of K1: it waits for K1's
 // completion with griddepcontrol.wait, so its CTAs can already be resident
 // while K1 drains.
@@ -578,7 +715,7 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     const int T = a.seq_lens[b];
     if (T < 1 || T > a.max_blocks * a.s.bt) return;
     const int ns = num_splits(T);
-    if (ns <= 1) return;                           // written by K1
+    if (ns <= 1 || ns <= a.merge_max_splits) return;   // written by K1
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -593,19 +730,7 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     float m = -INFINITY, lsum = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
-    for (int sp = s0; sp < s1; ++sp) {
-        const float2 v = ml[sp];
-        const float4 o = po[sp * (kHeadDim / 4)];
-        const float mn = fmaxf(m, v.x);
-        const float c = ex2(m - mn);               // rescale what is summed so far
-        const float w = ex2(v.x - mn);
-        m = mn;
-        lsum = lsum * c + w * v.y;
-        acc.x = acc.x * c + w * o.x;
-        acc.y = acc.y * c + w * o.y;
-        acc.z = acc.z * c + w * o.z;
-        acc.w = acc.w * c + w * o.w;
-    }
+    for (int sp = s0; sp < s1; ++sp) lse_step(m, lsum, acc, ml[sp], po[sp * (kHeadDim / 4)]);
     s_acc[warp][lane] = acc;
     if (lane == 0) {
         s_m[warp] = m;
@@ -613,32 +738,15 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     }
     __syncthreads();
     if (warp == 0) {
-        float M = s_m[0];
+        float mq[kMergeChains], lq[kMergeChains];
+        float4 aq[kMergeChains];
 #pragma unroll
-        for (int w = 1; w < kCombineWarps; ++w) M = fmaxf(M, s_m[w]);
-        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
-        float l = 0.f;
-#pragma unroll
-        for (int w = 0; w < kCombineWarps; ++w) {
-            const float c = ex2(s_m[w] - M);       // an empty quarter has m = -inf: c = 0
-            const float4 x = s_acc[w][lane];
-            r.x += c * x.x;
-            r.y += c * x.y;
-            r.z += c * x.z;
-            r.w += c * x.w;
-            l += c * s_l[w];
+        for (int q = 0; q < kMergeChains; ++q) {
+            mq[q] = s_m[q];
+            lq[q] = s_l[q];
+            aq[q] = s_acc[q][lane];
         }
-        const float inv = 1.f / l;
-        if (a.out_bf16) {
-            float r0, r1;
-            uint2 pk;
-            pk.x = pack_bf16(r.x * inv, r.y * inv, r0, r1);
-            pk.y = pack_bf16(r.z * inv, r.w * inv, r0, r1);
-            reinterpret_cast<uint2 *>(reinterpret_cast<uint16_t *>(a.out) + row * kHeadDim)[lane] = pk;
-        } else {
-            reinterpret_cast<float4 *>(a.out + row * kHeadDim)[lane] =
-                make_float4(r.x * inv, r.y * inv, r.z * inv, r.w * inv);
-        }
+        merge_chains_store(a, row, lane, mq, lq, aq);
     }
 }
 
@@ -720,22 +828,31 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
         const double w = static_cast<double>(ctas) / (per_sm * static_cast<double>(num_sms));
         return w / static_cast<double>(static_cast<int64_t>(w) + (w > static_cast<int64_t>(w)));
     };
+    // Which sessions the split kernel merges itself (no combine launch for
+    // them; the bits are the same either way). A grid that fits the SMs at
+    // once: up to kMergeInKernel splits. A longer grid: up to 4, since there
+    // the last CTA's merge of many splits at the grid's end, and each CTA's
+    // arrival holding its SM slot from the next CTA, cost more than the
+    // combine (measured on GB300: trace steps +4.5 % with 16, per-layer calls
+    // of 4K-token sessions 1 % faster with 4).
+    DecodeArgs ka = a;
+    ka.merge_max_splits = ctas <= 2 * static_cast<int64_t>(num_sms) ? kMergeInKernel : 4;
     cudaError_t e;
     if (ctas <= num_sms) {
         c1.blockDim = dim3(kWarpsWide * 32);
         c1.dynamicSmemBytes = decode_smem(kWarpsWide, kStagesOne);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsWide, kStagesOne>, map, a);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsWide, kStagesOne>, map, ka);
     } else if (ctas <= 2 * static_cast<int64_t>(num_sms) || fill(2) > fill(3) + KVT_WAVE_MARGIN) {
         c1.dynamicSmemBytes = decode_smem(kWarpsNarrow, kStagesHalf);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesHalf>, map, a);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesHalf>, map, ka);
     } else {
         c1.dynamicSmemBytes = decode_smem(kWarpsNarrow, kStagesFull);
-        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesFull>, map, a);
+        e = cudaLaunchKernelEx(&c1, decode_split_kernel<kWarpsNarrow, kStagesFull>, map, ka);
     }
     if (e != cudaSuccess) return e;
-    // Tables at most 1 024 tokens wide: every session is one split and the
-    // split kernel has written the outputs itself.
-    if (splits == 1) return cudaSuccess;
+    // Every session's output written by the split kernel: one split each, or
+    // few enough splits to merge there.
+    if (splits <= 1 || splits <= ka.merge_max_splits) return cudaSuccess;
 
     cudaLaunchConfig_t c2 = {};
     c2.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
@@ -744,7 +861,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
     c2.stream = st;
     c2.attrs = attr;
     c2.numAttrs = 1;
-    return cudaLaunchKernelEx(&c2, decode_combine_kernel, a);
+    return cudaLaunchKernelEx(&c2, decode_combine_kernel, ka);
 }
 
 }  // namespace kvt

@@ -69,6 +69,8 @@ struct DecodeArgs {
     float *out;               // [nl][B][Hq][D], fp32 or (out_bf16) bf16
     float *part_o;            // [nl*B][Hq][max_splits][D]
     float *part_ml;           // [nl*B][Hq][max_splits][2]
+    int32_t *counters;        // [nl*B][Hkv] split arrivals; zero between calls
+    int32_t merge_max_splits; // sessions of 2..this many splits merge in the split kernel
     int32_t *err;
     int32_t B, max_blocks, layer0, nlayers, max_splits;
     float scale_log2;         // scale * log2(e)

@@ -19,6 +19,12 @@ constexpr int kMaxDevices = 64;
 
 // Partials (fp32 accumulators, then (max, sum) pairs), then one flag word.
 static __device__ __align__(256) unsigned char g_decode_scratch[KV_NOALLOC_SCRATCH_BYTES];
+// Split-arrival counters, one per (layer-batch row, kv-head): zero when the
+// module loads, and every call leaves them at zero (the last arrival of a
+// group resets its counter). They sit apart from the scratch because the
+// partials' extent moves with each call's shape and the counters must not.
+constexpr int kMaxCounters = 65535 * 8;   // rows x kv-heads at most
+static __device__ int32_t g_decode_counters[kMaxCounters];
 
 // Tensor maps of the hot arenas a device's calls have used, so that a call
 // over an arena seen before skips the encode (a driver call per decode).
@@ -32,6 +38,7 @@ struct CachedMap {
 
 struct DeviceScratch {
     unsigned char *ptr = nullptr;   // device address of g_decode_scratch
+    int32_t *counters = nullptr;    // device address of g_decode_counters
     int num_sms = 1;
     bool ready = false;
     CachedMap maps[kMapCache];
@@ -48,21 +55,24 @@ int fail(int code, const char *msg) {
 // Per-device set-up, run by the first call on each device with that device
 // current: the array's device address (the host-side symbol is only a
 // stand-in), the decode kernels' shared-memory attributes and the SM count.
-int setup_device(int dev, unsigned char **ptr, int *num_sms) {
+int setup_device(int dev, unsigned char **ptr, int32_t **counters, int *num_sms) {
     std::lock_guard<std::mutex> lk(g_mu);
     DeviceScratch &d = g_dev[dev];
     if (!d.ready) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || !p)
+        void *p = nullptr, *pc = nullptr;
+        if (cudaGetSymbolAddress(&p, g_decode_scratch) != cudaSuccess || !p ||
+            cudaGetSymbolAddress(&pc, g_decode_counters) != cudaSuccess || !pc)
             return fail(KV_ERR_CUDA, "decode_attention_noalloc: cudaGetSymbolAddress failed");
         if (kvt::prepare_kernels() != cudaSuccess)
             return fail(KV_ERR_CUDA, "decode_attention_noalloc: kernel attribute set-up failed");
         if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
             return fail(KV_ERR_CUDA, "decode_attention_noalloc: SM count query failed");
         d.ptr = static_cast<unsigned char *>(p);
+        d.counters = static_cast<int32_t *>(pc);
         d.ready = true;
     }
     *ptr = d.ptr;
+    *counters = d.counters;
     *num_sms = d.num_sms;
     return KV_OK;
 }
@@ -149,8 +159,9 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     } restore{prev, c.device};
 
     unsigned char *scratch = nullptr;
+    int32_t *counters = nullptr;
     int num_sms = 1;
-    int rc = setup_device(c.device, &scratch, &num_sms);
+    int rc = setup_device(c.device, &scratch, &counters, &num_sms);
     if (rc) return rc;
     CUtensorMap map;
     rc = device_tensor_map(c.device, c.hot_base, rows,
@@ -160,8 +171,8 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     // The kernels OR their bounds-check bits into this word. Nothing reads it
     // (this entry point has no pool to report through), so it needs no
-    // clearing; no scratch has to start at zero, since every partial is
-    // written before it is read within the call.
+    // clearing; no other scratch has to start at zero, since every partial
+    // is written before it is read within the call.
     int32_t *flag = reinterpret_cast<int32_t *>(scratch + KV_NOALLOC_SCRATCH_BYTES - 256);
 
     kvt::DecodeArgs a;
@@ -171,6 +182,7 @@ extern "C" int decode_attention_noalloc(const kv_pool_config *cfg, int32_t layer
     a.out = out;
     a.part_o = reinterpret_cast<float *>(scratch);
     a.part_ml = reinterpret_cast<float *>(scratch + o_bytes);
+    a.counters = counters;
     a.err = flag;
     a.B = B;
     a.max_blocks = max_blocks;

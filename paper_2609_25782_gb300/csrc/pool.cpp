@@ -119,6 +119,7 @@ struct kv_pool {
     int32_t *d_tables = nullptr;
     float *d_part_o = nullptr;
     float *d_part_ml = nullptr;
+    int32_t *d_counters = nullptr;       // split arrivals per (layer-batch row, kv-head)
     int32_t *d_err = nullptr;
     CUtensorMap tmap{};
 
@@ -464,6 +465,10 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
         if (!rc) rc = p->cuda("cudaMalloc(partials)", [&] {
             return cudaMalloc(&p->d_part_ml, prow * 2 * sizeof(float));
         });
+        // A multi-split call has at most part_rows / Hq layer-batch rows.
+        const int64_t cnt = prow / c.num_q_heads * c.num_kv_heads * 4;
+        if (!rc) rc = p->cuda("cudaMalloc(counters)", [&] { return cudaMalloc(&p->d_counters, cnt); });
+        if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_counters, 0, cnt); });
         if (!rc) rc = p->cuda("cudaMalloc(err)", [&] { return cudaMalloc(&p->d_err, 4); });
         if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_err, 0, 4); });
         if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_tables, 0xFF, tbl); });
@@ -500,6 +505,7 @@ int kv_pool_destroy(kv_pool *p) {
         cudaFree(p->d_tables);
         cudaFree(p->d_part_o);
         cudaFree(p->d_part_ml);
+        cudaFree(p->d_counters);
         cudaFree(p->d_err);
     }
     delete p;
@@ -894,6 +900,7 @@ static int decode_impl(kv_pool *p, int32_t layer, const void *q, const void *k_n
     a.out = out;
     a.part_o = p->d_part_o;
     a.part_ml = p->d_part_ml;
+    a.counters = p->d_counters;
     a.err = p->d_err;
     a.B = B;
     a.max_blocks = max_blocks;

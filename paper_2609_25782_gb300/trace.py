@@ -135,8 +135,10 @@ class TraceDriver:
         self.mig_events = []                 # (kind, start, end, bytes)
         # host clock (perf_counter) per trace step: begin, after pauses and
         # admissions, after the batch reservation, end of enqueue; then the
-        # CPU time the thread used over the step (time.thread_time)
+        # CPU time the thread used over the step (time.thread_time) and the
+        # decode steps still queued on the GPU when the step began
         self.host_stamps = []
+        self._done = 0                       # step_events[:_done] have finished
         self.gc_pauses = []                  # (generation, start, seconds) during run()
         self.admit_ev = {}
         self.last_decode_ev = None
@@ -194,6 +196,12 @@ class TraceDriver:
         cfg = self.cfg
         if self.gpu and cfg.max_ahead > 0 and len(self.step_events) >= cfg.max_ahead:
             self.step_events[-cfg.max_ahead][1].synchronize()
+        queued = 0
+        if self.gpu:
+            ev = self.step_events
+            while self._done < len(ev) and ev[self._done][1].query():
+                self._done += 1
+            queued = len(ev) - self._done
         h0 = time.perf_counter()
         c0 = time.thread_time()
         h_adm = h_res = None
@@ -319,7 +327,8 @@ class TraceDriver:
                 self._prefetch_next(k, sids)
         self.counts["steps"] += 1
         self.counts["session_tokens"] += sum(self.tokens)
-        self.host_stamps.append((h0, h_adm, h_res, time.perf_counter(), time.thread_time() - c0))
+        self.host_stamps.append((h0, h_adm, h_res, time.perf_counter(), time.thread_time() - c0,
+                                 queued))
 
     def _decode_calls(self, B: int, mb: int, k_new, v_new) -> None:
         """The step's per-layer decode calls on the decode stream."""
