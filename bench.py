@@ -920,7 +920,7 @@ def main():
                     help="cap on migration-kernel CTAs during the trace (0: none)")
     ap.add_argument("--only-trace", action="store_true",
                     help="run only the agentic trace (simple and residency modes)")
-    ap.add_argument("--trace-max-ahead", type=int, default=20,
+    ap.add_argument("--trace-max-ahead", type=int, default=30,
                     help="trace: steps the host may run ahead of the GPU (0: unbounded)")
     ap.add_argument("--trace-no-graphs", action="store_true",
                     help="trace: launch each step's decode calls directly (no CUDA graphs)")

@@ -63,9 +63,10 @@ class TraceConfig:
     # The host issues step k only after step k - max_ahead has finished on the
     # GPU; 0: never waits. The queued steps absorb host stalls (a descheduled
     # thread on a shared machine). The CUDA launch queue holds about 1 000
-    # launches (about ten steps of direct calls, about thirty replayed steps);
-    # a launch that waits for queue space can itself stall the host.
-    max_ahead: int = 20
+    # launches: about ten steps of direct calls; thirty replayed steps fit
+    # (measured: no launch waited for queue space). A launch that waits for
+    # queue space can itself stall the host.
+    max_ahead: int = 30
 
 
 @dataclass
