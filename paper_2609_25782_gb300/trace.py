@@ -304,8 +304,10 @@ class TraceDriver:
                 if g is not None:
                     with self._torch.cuda.stream(self.dstream):
                         g.replay()
+                    end.record(self.dstream)
                 else:
                     self._decode_calls(B, mb, k_new, v_new)
+                    end.record(self.dstream)
                     if cfg.graphs:               # record it for the next step of this shape
                         g = self._torch.cuda.CUDAGraph()
                         with self._torch.cuda.stream(self.dstream):
@@ -313,7 +315,6 @@ class TraceDriver:
                             self._decode_calls(B, mb, k_new, v_new)
                             g.capture_end()
                         self.graphs[(B, mb)] = g
-                end.record(self.dstream)
                 self.last_decode_ev = end
                 self.step_events.append((start, end, B, sum(self.tokens[i] for i in members)))
                 self.step_index.append(k)
