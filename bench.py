@@ -239,21 +239,25 @@ def run_decode(args, ws, rank):
 
     # End to end through the C ABI with host buffers: every step copies its
     # Q, block tables and seq_lens from pinned host memory and reads its
-    # outputs back. Inputs and outputs are double-buffered so that step k+1's
-    # upload and step k's read-back run on a copy stream while step k decodes.
+    # outputs back. Inputs and outputs rotate through NB buffers so that step
+    # k+1's upload and step k's read-back run on a copy stream while step k
+    # decodes, and the host may issue up to NB steps (about 50 ms of GPU work,
+    # about 500 launches: well inside the CUDA launch queue) before it waits
+    # for a read-back, which a host stall of tens of ms then does not drain.
+    NB = 5
     cs = torch.cuda.Stream(device=dev)
     q_h = torch.empty(q.shape, dtype=q.dtype).pin_memory()
     q_h.copy_(q.cpu())
     tab_h = torch.as_tensor(tables_h).pin_memory()
     len_h = torch.as_tensor(lens.astype(np.int32)).pin_memory()
-    out_h = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
-    q_d = [torch.empty_like(q) for _ in range(2)]
-    tab_d = [torch.empty_like(tables) for _ in range(2)]
-    len_d = [torch.empty_like(lens_d) for _ in range(2)]
-    out_d = [torch.empty_like(out) for _ in range(2)]
-    up_done = [torch.cuda.Event() for _ in range(2)]
-    dec_done = [torch.cuda.Event() for _ in range(2)]
-    down_done = [torch.cuda.Event() for _ in range(2)]
+    out_h = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(NB)]
+    q_d = [torch.empty_like(q) for _ in range(NB)]
+    tab_d = [torch.empty_like(tables) for _ in range(NB)]
+    len_d = [torch.empty_like(lens_d) for _ in range(NB)]
+    out_d = [torch.empty_like(out) for _ in range(NB)]
+    up_done = [torch.cuda.Event() for _ in range(NB)]
+    dec_done = [torch.cuda.Event() for _ in range(NB)]
+    down_done = [torch.cuda.Event() for _ in range(NB)]
     for ev in up_done + dec_done + down_done:
         ev.record(cs)
 
@@ -268,14 +272,14 @@ def run_decode(args, ws, rank):
     def e2e_run(nsteps):
         upload(0)
         for k in range(nsteps):
-            buf = k % 2
-            if k >= 2:
-                # the host consumes step k-2's result before issuing step k, as a
-                # serving loop would; a host running further ahead fills the CUDA
-                # launch queue, where a launch waiting for room can stall it
+            buf = k % NB
+            if k >= NB:
+                # the host consumes step k-NB's result before issuing step k, as a
+                # serving loop would; a host running much further ahead fills the
+                # CUDA launch queue, where a launch waiting for room can stall it
                 down_done[buf].synchronize()
             if k + 1 < nsteps:
-                upload(buf ^ 1)
+                upload((k + 1) % NB)
             stream.wait_event(up_done[buf])
             stream.wait_event(down_done[buf])     # this output buffer was read back
             for l in range(L):
@@ -286,7 +290,7 @@ def run_decode(args, ws, rank):
                 cs.wait_event(dec_done[buf])
                 out_h[buf].copy_(out_d[buf], non_blocking=True)
                 down_done[buf].record(cs)
-        stream.wait_event(down_done[(nsteps - 1) % 2])
+        stream.wait_event(down_done[(nsteps - 1) % NB])
 
     e2e_run(max(1, args.warmup // 2))
     torch.cuda.synchronize()
