@@ -698,6 +698,24 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
     for (int h = warp; h < G; h += kWarps) merge_head_in_kernel(a, row_base + h, nsplit, lane);
 }
 
+// K2 for tables of at most kMergeInKernel splits: one warp per (layer-batch
+// row, q-head), four per CTA, folding the four chains side by side from
+// registers (merge_head_in_kernel), so no shared memory or CTA barrier sits
+// between its loads and its store.
+__global__ void __launch_bounds__(128) decode_combine_small_kernel(const DecodeArgs a) {
+    asm volatile("griddepcontrol.launch_dependents;");   // a following overlapped call
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * 4 + (threadIdx.x >> 5);
+    if (row >= static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq) return;
+    const int b = static_cast<int>((row / a.s.Hq) % a.B);
+    // seq_lens is read before the wait, as K1 reads it (no decode kernel writes it)
+    const int T = a.seq_lens[b];
+    if (T < 1 || T > a.max_blocks * a.s.bt) return;
+    const int ns = num_splits(T);
+    if (ns <= 1 || ns <= a.merge_max_splits) return;   // written by K1
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    merge_head_in_kernel(a, row, ns, threadIdx.x & 31);
+}
+
 // K2: one CTA (4 warps) per (layer-batch row, q-head) of a session of more
 // than kMergeInKernel splits. Warp w folds chain w, the contiguous quarter
 // [w*ns/4, (w+1)*ns/4) of the splits (split order), then warp 0 merges the
@@ -854,13 +872,18 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
     // few enough splits to merge there.
     if (splits <= 1 || splits <= ka.merge_max_splits) return cudaSuccess;
 
+    const int64_t rows = static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq;
     cudaLaunchConfig_t c2 = {};
-    c2.gridDim = dim3(static_cast<unsigned>(static_cast<int64_t>(a.nlayers) * a.B * a.s.Hq));
     c2.blockDim = dim3(kCombineWarps * 32);
     c2.dynamicSmemBytes = 0;
     c2.stream = st;
     c2.attrs = attr;
     c2.numAttrs = 1;
+    if (splits <= kMergeInKernel) {
+        c2.gridDim = dim3(static_cast<unsigned>((rows + 3) / 4));
+        return cudaLaunchKernelEx(&c2, decode_combine_small_kernel, ka);
+    }
+    c2.gridDim = dim3(static_cast<unsigned>(rows));
     return cudaLaunchKernelEx(&c2, decode_combine_kernel, ka);
 }
 
