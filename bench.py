@@ -309,12 +309,12 @@ def run_decode(args, ws, rank):
 
     # Launches per call, as the library decides them: the split kernel, plus
     # the combine when a session of the table's width can have more splits
-    # than the split kernel merges itself (16 when the grid of splits x
-    # kv-heads x rows fits the SMs at once, else 4).
+    # than the split kernel merges itself (4 in a grid of splits x kv-heads x
+    # rows of at least 8 CTAs per SM, else none).
     from paper_2609_25782_gb300 import kvtier
     splits = kvtier.kv_decode_splits(max_blocks * BT)
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    in_kernel = 16 if splits * HKV * B2 <= 2 * sms else 4
+    in_kernel = 4 if splits * HKV * B2 >= 8 * sms else 0
     per_call = 1 if splits <= max(1, in_kernel) else 2
     res = {
         "graph": graph is not None, "launches_per_call": per_call,

@@ -5,13 +5,14 @@
 //                          staged by TMA (cp.async.bulk.tensor, 128-byte
 //                          swizzle) into a per-warp mbarrier ring, and the
 //                          group-by-tile products run on mma.sync bf16.
-//                          The last CTA of a session's kv-head to finish
-//                          merges its splits (log-sum-exp in a fixed order)
-//                          when they are few: up to 16 in a grid that fits
-//                          the SMs at once, up to 4 in a longer one.
-//   decode_combine_kernel  the same merge for the other multi-split
-//                          sessions, launched as a programmatic dependent of
-//                          the split kernel when the table width allows them.
+//                          In a long grid, the last CTA of a kv-head of a
+//                          session of at most 4 splits to finish merges them
+//                          (log-sum-exp in a fixed order).
+//   decode_combine_small_kernel, decode_combine_kernel
+//                          the same merge for the other multi-split sessions
+//                          (one warp per query head from registers, up to 16
+//                          splits; else four warps per head), launched as a
+//                          programmatic dependent of the split kernel.
 //
 // Hot pool: hot[NB][L][2][Hkv][bt][128] bf16. A (block, layer, K|V, head)
 // run is bt rows of 256 B, row = ((blk*L + l)*2 + kv)*Hkv + g)*bt + slot. The
@@ -31,13 +32,15 @@ namespace {
 constexpr int kCombineWarps = 4;
 // The merge of a session's splits folds four chains (contiguous quarters of
 // the splits, in split order) and then merges the chains in order; that order
-// depends on the split count only, whichever kernel runs it. The split
-// kernel's last CTA of a (row, kv-head) can take up to kMergeInKernel splits
-// (four per chain).
+// depends on the split count only, whichever kernel runs it. One warp merges
+// up to kRegMergeMax splits from registers (four per chain); the split kernel
+// merges sessions of up to kSplitKernelMerge splits itself in long grids.
 constexpr int kMergeChains = 4;
-constexpr int kMergeInKernel = 16;
-static_assert(kCombineWarps == kMergeChains && kMergeInKernel == kMergeChains * 4,
-              "four splits per chain in the split kernel, one chain per combine warp");
+constexpr int kRegMergeMax = 16;
+constexpr int kSplitKernelMerge = 4;
+static_assert(kCombineWarps == kMergeChains && kRegMergeMax == kMergeChains * 4 &&
+                  kSplitKernelMerge <= kRegMergeMax,
+              "four splits per chain in a register merge, one chain per combine warp");
 constexpr int kTileBytes = 8192;           // K 4 KiB + V 4 KiB
 constexpr int kHalfBytes = 2048;           // 16 rows x 128 B (64 dims)
 // The plan of one split: its tiles are dealt round robin to kAccs running
@@ -242,7 +245,7 @@ __device__ __forceinline__ void merge_chains_store(const DecodeArgs &a, int64_t 
 // the loads need no guard): lane t loads split t's (m, l), shared by shuffle,
 // and each lane its 4 dims of every split's accumulator. The partials come
 // from L2 (.cg), written there by other SMs.
-__device__ __forceinline__ void merge_head_in_kernel(const DecodeArgs &a, int64_t row, int ns,
+__device__ __forceinline__ void merge_head_regs(const DecodeArgs &a, int64_t row, int ns,
                                                      int lane) {
     const int64_t base = row * a.max_splits;
     const float2 mine = __ldcg(reinterpret_cast<const float2 *>(a.part_ml) + base +
@@ -286,7 +289,8 @@ __device__ __forceinline__ void merge_head_in_kernel(const DecodeArgs &a, int64_
 //   O^T[128 x 8] += V^T[128 x 16] . P^T[16 x 8]     8 x mma, P^T via movmatrix
 // The accumulators merge in shared memory in accumulator order; a one-split
 // session writes its normalised output, others write (m, l, acc) partials,
-// which the group's last CTA to finish merges when there are at most 16.
+// which the group's last CTA to finish merges when the launch allows it
+// (a.merge_max_splits), else the combine kernel.
 // ---------------------------------------------------------------------------
 struct AccState {
     float m0, m1;   // running max, heads 2(lane%4) and +1 (log2 units)
@@ -695,12 +699,12 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
     __syncthreads();
     if (!s_last) return;
 #pragma unroll 1
-    for (int h = warp; h < G; h += kWarps) merge_head_in_kernel(a, row_base + h, nsplit, lane);
+    for (int h = warp; h < G; h += kWarps) merge_head_regs(a, row_base + h, nsplit, lane);
 }
 
-// K2 for tables of at most kMergeInKernel splits: one warp per (layer-batch
+// K2 for tables of at most kRegMergeMax splits: one warp per (layer-batch
 // row, q-head), four per CTA, folding the four chains side by side from
-// registers (merge_head_in_kernel), so no shared memory or CTA barrier sits
+// registers (merge_head_regs), so no shared memory or CTA barrier sits
 // between its loads and its store.
 __global__ void __launch_bounds__(128) decode_combine_small_kernel(const DecodeArgs a) {
     asm volatile("griddepcontrol.launch_dependents;");   // a following overlapped call
@@ -713,11 +717,11 @@ __global__ void __launch_bounds__(128) decode_combine_small_kernel(const DecodeA
     const int ns = num_splits(T);
     if (ns <= 1 || ns <= a.merge_max_splits) return;   // written by K1
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    merge_head_in_kernel(a, row, ns, threadIdx.x & 31);
+    merge_head_regs(a, row, ns, threadIdx.x & 31);
 }
 
-// K2: one CTA (4 warps) per (layer-batch row, q-head) of a session of more
-// than kMergeInKernel splits. Warp w folds chain w, the contiguous quarter
+// K2 for wider tables: one CTA (4 warps) per (layer-batch row, q-head) of a
+// multi-split session the split kernel did not merge. Warp w folds chain w, the contiguous quarter
 // [w*ns/4, (w+1)*ns/4) of the splits (split order), then warp 0 merges the
 // four chains in order. The result depends only on the partials
 // and ns. Launched as a programmatic dependent of K1: it waits for K1's
@@ -846,15 +850,17 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
         const double w = static_cast<double>(ctas) / (per_sm * static_cast<double>(num_sms));
         return w / static_cast<double>(static_cast<int64_t>(w) + (w > static_cast<int64_t>(w)));
     };
-    // Which sessions the split kernel merges itself (no combine launch for
-    // them; the bits are the same either way). A grid that fits the SMs at
-    // once: up to kMergeInKernel splits. A longer grid: up to 4, since there
-    // the last CTA's merge of many splits at the grid's end, and each CTA's
-    // arrival holding its SM slot from the next CTA, cost more than the
-    // combine (measured on GB300: trace steps +4.5 % with 16, per-layer calls
-    // of 4K-token sessions 1 % faster with 4).
+    // Which sessions the split kernel merges itself (the bits are the same
+    // either way): those of up to kSplitKernelMerge splits, in grids of at
+    // least 8 CTAs per SM. There, many groups finish at different times and
+    // their merges spread over the grid. In shorter grids each CTA's arrival
+    // (an atomic round trip holding its SM slot) and the tail merges cost more
+    // than the combine launch (measured on GB300 against merging everything in
+    // the combine: 256 x 4K-token sessions per layer +1.3 %, 8 x 4K all
+    // layers +1.6 %; one 4K- or 16K-token session per layer -7 % / -5 % and
+    // 32 x 4K -5 % when shorter grids merged too).
     DecodeArgs ka = a;
-    ka.merge_max_splits = ctas <= 2 * static_cast<int64_t>(num_sms) ? kMergeInKernel : 4;
+    ka.merge_max_splits = ctas >= 8 * static_cast<int64_t>(num_sms) ? kSplitKernelMerge : 0;
     cudaError_t e;
     if (ctas <= num_sms) {
         c1.blockDim = dim3(kWarpsWide * 32);
@@ -879,7 +885,7 @@ cudaError_t launch_decode(const CUtensorMap &map, const DecodeArgs &a, int num_s
     c2.stream = st;
     c2.attrs = attr;
     c2.numAttrs = 1;
-    if (splits <= kMergeInKernel) {
+    if (splits <= kRegMergeMax) {
         c2.gridDim = dim3(static_cast<unsigned>((rows + 3) / 4));
         return cudaLaunchKernelEx(&c2, decode_combine_small_kernel, ka);
     }

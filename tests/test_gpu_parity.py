@@ -169,34 +169,42 @@ def test_ring_depths_bit_identical(pkg):
 
 
 def test_merge_paths_bit_identical(pkg):
-    """A session of several splits is merged either by the split kernel (the
-    last CTA of each of its kv-heads to finish: up to 16 splits when the grid
-    fits the SMs at once, up to 4 in a longer grid) or by the combine kernel.
-    Both fold the same four chains of splits in the same order, so a
-    session's output is the same bits whichever merges it. The calls reuse
-    batch rows for sessions of other split counts, which also checks that
-    every call leaves its split-arrival counters at zero."""
+    """A session of several splits is merged by the split kernel (the last
+    CTA of each of its kv-heads to finish; sessions of up to 4 splits in a
+    grid of at least 8 CTAs per SM) or by a combine kernel (one warp per
+    query head from registers for tables of up to 16 splits, else four warps
+    per head). All fold the same four chains of splits in the same order, so
+    a session's output is the same bits whichever merges it. The all-layer
+    calls reuse batch rows for sessions of other split counts, which also
+    checks that every call leaves its split-arrival counters at zero."""
     lens = [1500, 4000, 4500, 8000, 12800, 16000, 3001]   # 2, 4, 5, 8, 13, 16, 3 splits
     L = 4
     pool, sess, tables, q = direct_case(pkg, lens, L=L, seed=31, max_batch=L * len(lens))
     n = len(lens)
-    # per layer, all sessions: 16 x 4 x 7 = 448 CTAs (more than two per SM):
-    # sessions of up to 4 splits merge in the split kernel, the others in the combine
+    # per layer, all sessions: 16 x 4 x 7 = 448 CTAs: every session merges in the
+    # register combine (tables of 1 000 blocks, 16 splits at most)
     batch = np.concatenate([gpu_decode(pool, l, q, tables, lens) for l in range(L)])
-    # one session per call: at most 64 CTAs, every session merges in the split kernel
+    # one session per call, in tables 2 048 blocks wide (32K tokens: 16 splits) and
+    # 2 112 blocks wide (17 splits: the four-warp combine)
     alone = np.zeros_like(batch)
+    wide = np.pad(tables, ((0, 0), (0, 2112 - tables.shape[1])), constant_values=-1)
+    alone_wide = np.zeros_like(batch)
     for i in range(n):
         qi = q[:, i:i + 1].contiguous()
         for l in range(L):
             alone[l, i] = gpu_decode(pool, l, qi, tables[i:i + 1], lens[i:i + 1])[0, 0]
+            alone_wide[l, i] = gpu_decode(pool, l, qi, wide[i:i + 1], lens[i:i + 1])[0, 0]
     # rows reversed, so each row holds a session of another split count than before
     rev = list(reversed(range(n)))
     qr = q[:, rev].contiguous()
     back = np.concatenate([gpu_decode(pool, l, qr, tables[rev], [lens[i] for i in rev])
                            for l in range(L)])[:, rev]
-    # all layers in one call: 16 x 4 x 28 = 1 792 CTAs
+    # all layers in one call: 16 x 4 x 28 = 1 792 CTAs, at least 8 per SM: the split
+    # kernel merges the sessions of up to 4 splits (1 500, 3 001 and 4 000 tokens),
+    # first with these rows, then with the rows reversed
     whole = gpu_decode(pool, -1, q, tables, lens)
-    for other in (alone, back, whole):
+    whole_back = gpu_decode(pool, -1, qr, tables[rev], [lens[i] for i in rev])[:, rev]
+    for other in (alone, alone_wide, back, whole, whole_back):
         assert np.array_equal(batch.view(np.int64), other.view(np.int64))
     ref = oracle.paged_decode(host_hot(pool, 31, sess, lens, tables), q.cpu().view(torch.int16)
                               .numpy().view(np.uint16), tables, lens, 1 / math.sqrt(128), 32)
