@@ -631,51 +631,49 @@ __global__ void __launch_bounds__(kWarps * 32, kWarps == kWarpsNarrow && kStages
     }
     __syncthreads();
 
-    // Merge the accumulators in order; a thread handles (head, 8 dims).
+    // Merge the accumulators in order; a thread handles (head, 4 dims), so a
+    // warp reads one head's row of each state as 32 consecutive float4.
     auto acc_base = [&](int v) {
         return reinterpret_cast<const float *>(smem + (v % kWarps) * kStages * kTileBytes) +
                (v / kWarps) * kAccFloats;
     };
     const int64_t row_base = static_cast<int64_t>(lb) * sh.Hq + g * G;
-    for (int e = threadIdx.x; e < G * (kHeadDim / 8); e += blockDim.x) {
-        const int h = e / (kHeadDim / 8);
-        const int d0 = (e % (kHeadDim / 8)) * 8;
+    for (int e = threadIdx.x; e < G * (kHeadDim / 4); e += blockDim.x) {
+        const int h = e / (kHeadDim / 4);
+        const int d0 = (e % (kHeadDim / 4)) * 4;
         float M = -INFINITY;
 #pragma unroll
         for (int v = 0; v < kAccs; ++v) M = fmaxf(M, acc_base(v)[kMaxGroup * kOStride + h]);
-        float lsum = 0.f, acc[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+        float lsum = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int v = 0; v < kAccs; ++v) {
             const float *wsv = acc_base(v);
             const float *wmv = wsv + kMaxGroup * kOStride;
             const float sc = ex2(wmv[h] - M);      // an accumulator with no tile: m = -inf, 0
             lsum += sc * wmv[8 + h];
-#pragma unroll
-            for (int c = 0; c < 8; ++c) acc[c] += sc * wsv[h * kOStride + d0 + c];
+            const float4 x = *reinterpret_cast<const float4 *>(wsv + h * kOStride + d0);
+            acc.x += sc * x.x;
+            acc.y += sc * x.y;
+            acc.z += sc * x.z;
+            acc.w += sc * x.w;
         }
         if (nsplit == 1) {
             const float inv = 1.f / lsum;
             if (a.out_bf16) {
-                uint4 pk;
+                uint2 pk;
                 float r0, r1;
-                pk.x = pack_bf16(acc[0] * inv, acc[1] * inv, r0, r1);
-                pk.y = pack_bf16(acc[2] * inv, acc[3] * inv, r0, r1);
-                pk.z = pack_bf16(acc[4] * inv, acc[5] * inv, r0, r1);
-                pk.w = pack_bf16(acc[6] * inv, acc[7] * inv, r0, r1);
-                *reinterpret_cast<uint4 *>(reinterpret_cast<uint16_t *>(a.out) +
+                pk.x = pack_bf16(acc.x * inv, acc.y * inv, r0, r1);
+                pk.y = pack_bf16(acc.z * inv, acc.w * inv, r0, r1);
+                *reinterpret_cast<uint2 *>(reinterpret_cast<uint16_t *>(a.out) +
                                            (row_base + h) * kHeadDim + d0) = pk;
             } else {
-                float4 *dst = reinterpret_cast<float4 *>(a.out + (row_base + h) * kHeadDim + d0);
-                dst[0] = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
-                dst[1] = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
+                *reinterpret_cast<float4 *>(a.out + (row_base + h) * kHeadDim + d0) =
+                    make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
             }
         } else {
             const int64_t prow = (row_base + h) * a.max_splits + split;
-            float4 *dst = reinterpret_cast<float4 *>(a.part_o + prow * kHeadDim + d0);
-            dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-            dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+            *reinterpret_cast<float4 *>(a.part_o + prow * kHeadDim + d0) = acc;
             if (d0 == 0) {
                 a.part_ml[prow * 2] = M;
                 a.part_ml[prow * 2 + 1] = lsum;
