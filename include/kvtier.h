@@ -380,16 +380,21 @@ int kv_pool_free_list(kv_pool *pool, int32_t *host_out, int64_t cap, int64_t *n)
 
 int kv_pool_get_stats(kv_pool *pool, kv_pool_stats *out);
 
-/* Bits of the device flag word that kernels set when their own checks fire. */
-#define KV_DEVICE_BAD_BLOCK 1   /* a block id outside the pool (access skipped)     */
-#define KV_DEVICE_BAD_LENGTH 2  /* seq_len < 1 or past its table row (row skipped) */
-#define KV_DEVICE_TIMEOUT 4     /* a tile wait gave up after 2 s (output undefined) */
+/* Bits of the device flag word that kernels set when their own checks fire,
+ * and (STALE_COUNTERS) what kv_pool_check_device finds in the workspace. */
+#define KV_DEVICE_BAD_BLOCK 1      /* a block id outside the pool (access skipped)     */
+#define KV_DEVICE_BAD_LENGTH 2     /* seq_len < 1 or past its table row (row skipped) */
+#define KV_DEVICE_TIMEOUT 4        /* a tile wait gave up after 2 s (output undefined) */
+#define KV_DEVICE_STALE_COUNTERS 8 /* split-arrival counters not at zero (reset)       */
 
 /* Synchronise the device and read the flags that kernels set when their own
  * bounds checks fire (a block id outside the pool, a length past a table
- * row, a wait that timed out); clears them. *flags = 0 means clean; a
- * non-zero value (KV_DEVICE_* bits) makes the call return
- * KV_ERR_DEVICE_CHECK. */
+ * row, a wait that timed out); clears them. Also checks that the decode
+ * workspace's split-arrival counters are back at zero, as every decode call
+ * leaves them; counters left non-zero (by decode calls that overlapped on
+ * the GPU) set KV_DEVICE_STALE_COUNTERS and are reset, so later calls are
+ * right again. *flags = 0 means clean; a non-zero value (KV_DEVICE_* bits)
+ * makes the call return KV_ERR_DEVICE_CHECK. Bookkeeping; no passage. */
 int kv_pool_check_device(kv_pool *pool, int32_t *flags);
 
 /* Cap the migration kernels (resume-unpack, pause-pack, evictions) at
@@ -413,6 +418,13 @@ int kv_pool_inject_cuda_failure(kv_pool *pool, int32_t n);
  * stays usable and kv_pool_check_device reports the flag. Disarms itself
  * after one call. */
 int kv_pool_inject_decode_timeout(kv_pool *pool, int32_t on);
+
+/* Test hook for the counter check: synchronises the device and sets the
+ * first split-arrival counter of the workspace to 1, as a decode call that
+ * overlapped another would leave it. The next kv_pool_check_device reports
+ * KV_DEVICE_STALE_COUNTERS and resets it. Errors: host-logic pool ->
+ * KV_ERR_BAD_STATE. */
+int kv_pool_inject_stale_counter(kv_pool *pool);
 
 /* Fixed size of the device scratch used by decode_attention_noalloc. */
 #define KV_NOALLOC_SCRATCH_BYTES (48ll << 20)

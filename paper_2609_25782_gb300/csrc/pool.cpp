@@ -120,6 +120,7 @@ struct kv_pool {
     float *d_part_o = nullptr;
     float *d_part_ml = nullptr;
     int32_t *d_counters = nullptr;       // split arrivals per (layer-batch row, kv-head)
+    int64_t counter_count = 0;
     int32_t *d_err = nullptr;
     CUtensorMap tmap{};
 
@@ -466,7 +467,8 @@ int kv_pool_create(const kv_pool_config *cfg, kv_pool **out) {
             return cudaMalloc(&p->d_part_ml, prow * 2 * sizeof(float));
         });
         // A multi-split call has at most part_rows / Hq layer-batch rows.
-        const int64_t cnt = prow / c.num_q_heads * c.num_kv_heads * 4;
+        p->counter_count = prow / c.num_q_heads * c.num_kv_heads;
+        const int64_t cnt = p->counter_count * 4;
         if (!rc) rc = p->cuda("cudaMalloc(counters)", [&] { return cudaMalloc(&p->d_counters, cnt); });
         if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_counters, 0, cnt); });
         if (!rc) rc = p->cuda("cudaMalloc(err)", [&] { return cudaMalloc(&p->d_err, 4); });
@@ -1327,8 +1329,22 @@ int kv_pool_check_device(kv_pool *p, int32_t *flags) {
         return cudaMemcpy(flags, p->d_err, 4, cudaMemcpyDeviceToHost);
     });
     if (!rc) rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_err, 0, 4); });
+    // Every decode call leaves the split-arrival counters at zero; any other
+    // value comes from calls that overlapped on the GPU.
+    std::vector<int32_t> cnt(static_cast<size_t>(p->counter_count));
+    if (!rc && !cnt.empty())
+        rc = p->cuda("cudaMemcpy", [&] {
+            return cudaMemcpy(cnt.data(), p->d_counters, cnt.size() * 4, cudaMemcpyDeviceToHost);
+        });
     if (rc) return rc;
-    if (*flags) return fail(KV_ERR_DEVICE_CHECK, "a kernel bounds check fired (flags " + std::to_string(*flags) + ")");
+    bool stale = false;
+    for (int32_t v : cnt) stale |= v != 0;
+    if (stale) {
+        rc = p->cuda("cudaMemset", [&] { return cudaMemset(p->d_counters, 0, cnt.size() * 4); });
+        if (rc) return rc;
+        *flags |= KV_DEVICE_STALE_COUNTERS;
+    }
+    if (*flags) return fail(KV_ERR_DEVICE_CHECK, "a device check fired (flags " + std::to_string(*flags) + ")");
     return KV_OK;
 }
 
@@ -1348,6 +1364,18 @@ int kv_pool_inject_decode_timeout(kv_pool *p, int32_t on) {
     if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
     p->inject_timeout = on != 0;
     return KV_OK;
+}
+
+int kv_pool_inject_stale_counter(kv_pool *p) {
+    if (!p) return fail(KV_ERR_INVALID_ARG, "null pool");
+    if (p->host_only) return fail(KV_ERR_BAD_STATE, "no device workspace on a host-logic pool");
+    DeviceGuard dg(p->cfg.device, true);
+    const int32_t one = 1;
+    int rc = p->cuda("cudaDeviceSynchronize", [&] { return cudaDeviceSynchronize(); });
+    if (!rc) rc = p->cuda("cudaMemcpy", [&] {
+        return cudaMemcpy(p->d_counters, &one, 4, cudaMemcpyHostToDevice);
+    });
+    return rc;
 }
 
 }  // extern "C"

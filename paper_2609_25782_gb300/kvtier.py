@@ -39,10 +39,11 @@ EXPORTS = [
     "kv_pool_inject_cuda_failure", "kv_last_error", "decode_attention_noalloc",
     "decode_attention_ex", "kv_pool_set_migration_limit", "kv_pool_batch_reserve",
     "decode_append_attention", "kv_pool_inject_decode_timeout", "kv_decode_splits",
-    "session_block_table_device", "kv_pool_prefetch",
+    "session_block_table_device", "kv_pool_prefetch", "kv_pool_inject_stale_counter",
 ]
 
 KV_DEVICE_BAD_BLOCK, KV_DEVICE_BAD_LENGTH, KV_DEVICE_TIMEOUT = 1, 2, 4
+KV_DEVICE_STALE_COUNTERS = 8
 
 KV_DECODE_OVERLAP_PREVIOUS = 1
 KV_DECODE_OUT_BF16 = 2
@@ -116,6 +117,7 @@ def _load():
         "kv_pool_check_device": [p, C.POINTER(i32)],
         "kv_pool_inject_cuda_failure": [p, i32],
         "kv_pool_inject_decode_timeout": [p, i32],
+        "kv_pool_inject_stale_counter": [p],
         "kv_pool_set_migration_limit": [p, i32],
         "kv_last_error": [],
         "decode_attention_noalloc": [C.POINTER(kv_pool_config), i32, p, p, p, i32, i32,
@@ -317,6 +319,10 @@ def kv_pool_check_device(pool: int) -> int:
 
 def kv_pool_inject_decode_timeout(pool: int, on: int = 1) -> None:
     _check(lib.kv_pool_inject_decode_timeout(pool, on), "kv_pool_inject_decode_timeout")
+
+
+def kv_pool_inject_stale_counter(pool: int) -> None:
+    _check(lib.kv_pool_inject_stale_counter(pool), "kv_pool_inject_stale_counter")
 
 
 def kv_pool_set_migration_limit(pool: int, max_ctas: int) -> None:

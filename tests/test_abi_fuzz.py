@@ -137,7 +137,13 @@ def test_decode_flags_and_arguments_rejected(kv):
     assert e.value.code == kv.KV_ERR_INVALID_ARG
     kv.kv_pool_inject_decode_timeout(pool, 1)          # armed, then disarmed: host state only
     kv.kv_pool_inject_decode_timeout(pool, 0)
+    with pytest.raises(kv.KVError) as e:               # no device workspace to touch
+        kv.kv_pool_inject_stale_counter(pool)
+    assert e.value.code == kv.KV_ERR_BAD_STATE
     kv.kv_pool_destroy(pool)
+    with pytest.raises(kv.KVError) as e:
+        kv.kv_pool_inject_stale_counter(None)
+    assert e.value.code == kv.KV_ERR_INVALID_ARG
     with pytest.raises(kv.KVError) as e:
         kv.kv_pool_inject_decode_timeout(None, 1)
     assert e.value.code == kv.KV_ERR_INVALID_ARG
