@@ -104,6 +104,16 @@ int main(void) {
         expect_code("device table row on a host-logic pool",
                     session_block_table_device(pool, s0, &dev_row, &nb), KV_ERR_BAD_STATE);
     }
+    {
+        int32_t flags = -1;
+        expect_code("device check on a host-logic pool", kv_pool_check_device(pool, &flags), KV_OK);
+        if (flags != 0) {
+            fprintf(stderr, "device check on a host-logic pool: flags %d\n", flags);
+            ++failures;
+        }
+        expect_code("stale-counter hook on a host-logic pool", kv_pool_inject_stale_counter(pool),
+                    KV_ERR_BAD_STATE);
+    }
     batch[1] = s0;
     expect_code("session twice in a batch",
                 kv_pool_batch_reserve(pool, batch, 2, NULL, 64, NULL, NULL), KV_ERR_INVALID_ARG);
