@@ -749,8 +749,22 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const DecodeArgs a)
     const int s1 = ((warp + 1) * ns) / kCombineWarps;
     float m = -INFINITY, lsum = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-    for (int sp = s0; sp < s1; ++sp) lse_step(m, lsum, acc, ml[sp], po[sp * (kHeadDim / 4)]);
+    // Batches of kCombineBatch splits: every load of a batch is issued before
+    // the first is folded (indices clamped into the quarter, no guards).
+    constexpr int kCombineBatch = 16;
+    for (int sb = s0; sb < s1; sb += kCombineBatch) {
+        float2 v[kCombineBatch];
+        float4 o[kCombineBatch];
+#pragma unroll
+        for (int j = 0; j < kCombineBatch; ++j) {
+            const int sp = min(sb + j, s1 - 1);
+            v[j] = ml[sp];
+            o[j] = po[sp * (kHeadDim / 4)];
+        }
+#pragma unroll
+        for (int j = 0; j < kCombineBatch; ++j)
+            if (sb + j < s1) lse_step(m, lsum, acc, v[j], o[j]);
+    }
     s_acc[warp][lane] = acc;
     if (lane == 0) {
         s_m[warp] = m;
